@@ -1,0 +1,538 @@
+"""Benchmark of the RS3-Prune hot path on one GB300 (or N, one process each).
+
+One *step* is the whole SAM2-shaped single-object sequence (60 frames): bank
+reset, the conditioning frame's commit and pointer rows, then for frames
+1..59 the read-side selection (Eq. 1/2/4/5), the pruned readout with the
+residual scatter (Eq. 6) and the write-pruned commit (Eq. 8).  All inputs
+(query grids, residual grids, memory-encoder K/V, masks) are resident in HBM
+when the timed region starts; together they exceed the 129 MB L2, so no flush
+is needed between steps.  The step is replayed from a CUDA graph.
+
+Printed: one JSON line (rank 0).  `--impl reference` times the CPU oracle on
+the host cores instead (a bounded sample of the same workload).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "pruned readout frames/s & TFLOP/s vs dense (1 GB300); bank-commit HBM GB/s"
+WORKLOAD = "sam2_1obj"
+KERNELS_PER_READOUT_FRAME = 8     # prior, energy, select, plan, readout, combine, commit plan, commit copy
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return p.get("hbm_gbs", 6800.0), p.get("bf16_tflops", 1900.0), \
+            p.get("bf16_tflops_sustained", 1700.0), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (one process per GPU; units are independent, so each
+# rank runs its own streams: weak scaling with no data-path collective)
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def aggregate(frames_per_rank, seconds_per_rank):
+    """Whole-job throughput: all frames of all ranks over the slowest rank."""
+    t = max(seconds_per_rank)
+    return sum(frames_per_rank) / t if t > 0 else 0.0, t
+
+
+def allgather_floats(vals, world):
+    if world == 1:
+        return [list(vals)]
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor(list(vals), dtype=torch.float64, device=dev)
+    out = [torch.zeros_like(t) for _ in range(world)]
+    dist.all_gather(out, t)
+    return [o.cpu().tolist() for o in out]
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower() in ("active", "1"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(max(smax)),
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------
+# the GPU arm
+# ---------------------------------------------------------------------------
+
+class DeviceSequence:
+    """All inputs of one sequence, resident on the device (and pinned on the
+    host for the end-to-end leg)."""
+
+    def __init__(self, w, dense: bool, device):
+        import torch
+        from paper_2608_22526_gb300 import synth
+        seq = synth.Sequence(w)
+        T = w.frames
+        ug = w.unit_group()
+
+        def dev(x):
+            if x.dtype == np.uint16:
+                return torch.from_numpy(x.view(np.int16)).view(torch.bfloat16)
+            return torch.from_numpy(np.ascontiguousarray(x))
+
+        z = [seq.z(t) for t in range(T)]
+        kv = [seq.kv_new(t) for t in range(T)]
+        masks = [seq.masks(t) for t in range(T)]
+        self.host = {
+            "z": dev(np.stack(z)).pin_memory(),
+            "x": dev(np.stack([zz[ug] for zz in z])).pin_memory(),
+            "k": dev(np.stack([a for a, _ in kv])).pin_memory(),
+            "v": dev(np.stack([b for _, b in kv])).pin_memory(),
+            "mask": torch.from_numpy(np.stack(masks)).pin_memory(),
+        }
+        if dense:
+            self.host["prev"] = torch.ones_like(self.host["mask"]).pin_memory()
+        else:
+            prev = np.concatenate([np.zeros((1,) + masks[0].shape, np.uint8), np.stack(masks[:-1])])
+            self.host["prev"] = torch.from_numpy(prev).pin_memory()
+        kp, vp = seq.pointers()
+        self.ptr = (dev(kp).to(device), dev(vp).to(device)) if w.n_ptr > 0 else None
+        self.dev = {k: v.to(device) for k, v in self.host.items()}
+        self.masks_np = masks
+        self.T = T
+
+    def h2d(self, stream):
+        import torch
+        with torch.cuda.stream(stream):
+            for k in ("z", "x", "k", "v", "mask", "prev"):
+                self.dev[k].copy_(self.host[k], non_blocking=True)
+
+    def bytes_in(self):
+        return sum(self.host[k].numel() * self.host[k].element_size()
+                   for k in ("z", "x", "k", "v", "mask", "prev"))
+
+
+def run_step(pipe, data, timers=None):
+    """One step: the whole sequence through the library (Algorithm 1's loop)."""
+    import torch
+    w = pipe.w
+    from paper_2608_22526_gb300 import rs3
+    rs3.rs3_bank_reset(pipe.bank, -1)
+    pipe.track.zero_()
+    D = data.dev
+    for t in range(data.T):
+        if t == 0 and w.n_cond > 0:
+            pipe.commit(D["k"][t], D["v"][t], D["mask"][t], 1)
+            if data.ptr is not None:
+                pipe.set_pointers(*data.ptr)
+            continue
+        if timers is not None:
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+            e[0].record()
+        pipe.select(D["z"][t], D["prev"][t])
+        if timers is not None:
+            e[1].record()
+        pipe.readout(D["z"][t], D["x"][t], D["x"][t])
+        if timers is not None:
+            e[2].record()
+        pipe.commit(D["k"][t], D["v"][t], D["mask"][t], 0)
+        if timers is not None:
+            e[3].record()
+            timers.append((t, e))
+
+
+def frame_work(w, counts, bank_lens, kw_lens):
+    """Algorithmic flops and bytes of one frame from the selected sizes."""
+    b = 2 if w.dtype == "bf16" else 4
+    flops = sum(4.0 * c * n * w.H * w.d for c, n in zip(counts, bank_lens))
+    commit_bytes = w.U * w.mn + sum(4.0 * L * w.D * b for L in kw_lens)
+    return flops, commit_bytes
+
+
+def work_model(pipe, data):
+    """Per readout frame: (counts, bank lengths) from one instrumented pass."""
+    import torch
+    from paper_2608_22526_gb300 import rs3
+    w = pipe.w
+    D = data.dev
+    rs3.rs3_bank_reset(pipe.bank, -1)
+    pipe.track.zero_()
+    out = []
+    for t in range(data.T):
+        if t == 0 and w.n_cond > 0:
+            pipe.commit(D["k"][t], D["v"][t], D["mask"][t], 1)
+            if data.ptr is not None:
+                pipe.set_pointers(*data.ptr)
+            continue
+        pipe.select(D["z"][t], D["prev"][t])
+        meta, _ = rs3.rs3_bank_read_meta(pipe.bank)
+        counts = pipe.count.cpu().tolist()
+        lens = meta[:, 7].tolist()
+        x = D["x"][t].clone()
+        pipe.readout(D["z"][t], x, x)
+        if pipe.dense:
+            kwl = [w.mn] * w.U
+        else:
+            kwl = [int(v) for v in data.masks_np[t].astype(bool).sum(axis=1)]
+        pipe.commit(D["k"][t], D["v"][t], D["mask"][t], 0)
+        out.append((t, counts, lens, kwl))
+    torch.cuda.synchronize()
+    return out
+
+
+def gpu_arm(args):
+    import torch
+    import torch.distributed as dist
+    rank, world, local = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    from paper_2608_22526_gb300 import synth
+    from paper_2608_22526_gb300.pipeline import Pipeline
+
+    w = synth.WORKLOADS[args.workload]
+    hbm, tc_burst, tc_sust, peak_src = _peaks()
+
+    def build(dense):
+        data = DeviceSequence(w, dense, device)
+        pipe = Pipeline(w, device=device, dense=dense)
+        return pipe, data
+
+    results = {}
+    for mode in (["pruned", "dense"] if not args.no_dense else ["pruned"]):
+        pipe, data = build(mode == "dense")
+        stream = torch.cuda.Stream()
+        with torch.cuda.stream(stream):
+            # warm-up (also sets kernel attributes before capture)
+            for _ in range(max(args.warmup, 1)):
+                run_step(pipe, data)
+            torch.cuda.synchronize()
+            work = work_model(pipe, data)
+            torch.cuda.synchronize()
+            # per-call timing pass (events on the launching stream)
+            timers = []
+            run_step(pipe, data, timers)
+            torch.cuda.synchronize()
+            sel_ms = [t[1][0].elapsed_time(t[1][1]) for t in timers]
+            rd_ms = [t[1][1].elapsed_time(t[1][2]) for t in timers]
+            cm_ms = [t[1][2].elapsed_time(t[1][3]) for t in timers]
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=stream):
+                run_step(pipe, data)
+            for _ in range(args.warmup):
+                graph.replay()
+            torch.cuda.synchronize()
+            if world > 1:
+                dist.barrier()
+            clocks = ClockSampler(local) if mode == "pruned" else None
+            if clocks:
+                clocks.start()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            e0.record()
+            for _ in range(args.steps):
+                graph.replay()
+            e1.record()
+            torch.cuda.synchronize()
+            dev_s = e0.elapsed_time(e1) / 1e3
+            clk = clocks.stop() if clocks else None
+            assert int(pipe.status.item()) == 0, "device status word set"
+            # end-to-end through the public API with host buffers
+            e2e_s = None
+            if mode == "pruned" and not args.no_e2e:
+                out_host = torch.empty_like(data.host["x"]).pin_memory()
+                for _ in range(2):
+                    data.h2d(stream)
+                    graph.replay()
+                    out_host.copy_(data.dev["x"], non_blocking=True)
+                torch.cuda.synchronize()
+                f0 = torch.cuda.Event(enable_timing=True)
+                f1 = torch.cuda.Event(enable_timing=True)
+                f0.record()
+                for _ in range(args.steps):
+                    data.h2d(stream)
+                    graph.replay()
+                    out_host.copy_(data.dev["x"], non_blocking=True)
+                f1.record()
+                torch.cuda.synchronize()
+                e2e_s = f0.elapsed_time(f1) / 1e3
+                e2e_bytes = (data.bytes_in(), out_host.numel() * out_host.element_size())
+        flops = [frame_work(w, c, n, k)[0] for (_, c, n, k) in work]
+        cbytes = [frame_work(w, c, n, k)[1] for (_, c, n, k) in work]
+        results[mode] = dict(dev_s=dev_s, e2e_s=e2e_s, clocks=clk, sel_ms=sel_ms, rd_ms=rd_ms,
+                             cm_ms=cm_ms, flops=flops, cbytes=cbytes,
+                             e2e_bytes=e2e_bytes if mode == "pruned" and e2e_s else None,
+                             counts=[c for (_, c, _, _) in work], lens=[n for (_, _, n, _) in work])
+        del graph, pipe, data
+        torch.cuda.empty_cache()
+
+    frames_per_step = w.frames * w.G
+    P = results["pruned"]
+    gathered = allgather_floats([P["dev_s"], P["e2e_s"] or 0.0], world)
+    value, tmax = aggregate([frames_per_step * args.steps] * world, [g[0] for g in gathered])
+    e2e_val = None
+    if P["e2e_s"]:
+        e2e_val, _ = aggregate([frames_per_step * args.steps] * world, [g[1] for g in gathered])
+    if rank != 0:
+        if world > 1:
+            dist.barrier()
+            dist.destroy_process_group()
+        return
+    rd_avg_ms = float(np.mean(P["rd_ms"]))
+    flops_avg = float(np.mean(P["flops"]))
+    achieved_tflops = flops_avg / (rd_avg_ms / 1e3) / 1e12
+    step_flops = sum(P["flops"])
+    traffic = _traffic_record(w)
+    line = {
+        "metric": METRIC,
+        "value": round(value, 2),
+        "unit": "frames/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(tmax / args.steps * 1e3, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": w.dtype,
+        "data": "synthetic (seeded SAM2-shaped drifting-ellipse sequence; no dataset)",
+        "config": {"workload": f"{w.name}: {w.m}x{w.n} grid, {w.H}x{w.d} heads, cond + {w.window} "
+                               f"recent write-pruned frames + {w.n_ptr} pointer rows, "
+                               f"{w.frames} frames per step, rho {w.rho}",
+                   "global_batch": world, "seq_len": w.frames,
+                   "parallelism": f"replicas x{world}",
+                   "l2": "inputs per step exceed L2 (no flush)",
+                   "timing": "CUDA graph of the whole sequence, CUDA events"},
+        "readout_tflops": round(step_flops * args.steps / (P["dev_s"]) / 1e12, 3),
+        "roofline": {"bound": "tensor", "achieved": round(achieved_tflops, 3),
+                     "peak": tc_burst, "unit": "TFLOP/s",
+                     "frac": round(achieved_tflops / tc_burst, 4),
+                     "traffic": traffic,
+                     "kernel": "rs3_memory_readout (plan + readout + combine)",
+                     "peak_source": f"bf16_tflops burst, {peak_src}"},
+        "commit_gbs": round(float(np.mean(P["cbytes"])) / (float(np.mean(P["cm_ms"])) / 1e3) / 1e9, 2),
+        "commit_frac_hbm": round(float(np.mean(P["cbytes"])) / (float(np.mean(P["cm_ms"])) / 1e3) / 1e9 / hbm, 4),
+        "select_ms": round(float(np.mean(P["sel_ms"])), 4),
+        "readout_ms": round(rd_avg_ms, 4),
+        "commit_ms": round(float(np.mean(P["cm_ms"])), 4),
+        "mean_queries": round(float(np.mean([sum(c) for c in P["counts"]])), 1),
+        "mean_bank_rows": round(float(np.mean([sum(n) for n in P["lens"]])), 1),
+        "clocks": P["clocks"],
+        "gpu_launches": (1 + (3 if w.n_ptr > 0 else 2) + (w.frames - (1 if w.n_cond > 0 else 0))
+                         * KERNELS_PER_READOUT_FRAME) * args.steps,
+    }
+    if "dense" in results:
+        Dn = results["dense"]
+        dense_fps = frames_per_step * args.steps / Dn["dev_s"]
+        line["dense"] = {"value": round(dense_fps, 2), "unit": "frames/s",
+                         "readout_tflops": round(sum(Dn["flops"]) * args.steps / Dn["dev_s"] / 1e12, 3),
+                         "readout_ms": round(float(np.mean(Dn["rd_ms"])), 4)}
+        line["speedup_vs_dense"] = round(value / dense_fps, 3) if world == 1 else None
+    if P["e2e_s"]:
+        line["e2e"] = {"value": round(e2e_val, 2), "unit": "frames/s",
+                       "h2d_bytes_per_step": int(P["e2e_bytes"][0]),
+                       "d2h_bytes_per_step": int(P["e2e_bytes"][1])}
+    if not args.no_cpu_baseline and world == 1:
+        line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_seconds)
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def _traffic_record(w):
+    """DRAM bytes per readout launch from a committed ncu capture, if the
+    readout sources have not changed since."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            rec = json.load(f)
+        if rec.get("source_hash") != readout_source_hash():
+            return None
+        return rec.get("per_launch_bytes", {}).get(w.name)
+    except Exception:
+        return None
+
+
+def readout_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_22526_gb300", "csrc")
+    for f in ("rs3_readout.cu", "rs3_readout_tc.cu", "rs3_readout_common.cuh"):
+        p = os.path.join(csrc, f)
+        if os.path.exists(p):
+            h.update(open(p, "rb").read())
+    return h.hexdigest()[:16]
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (baseline leg and the reference arm)
+# ---------------------------------------------------------------------------
+
+def oracle_frames(w, budget_s: float, threads: int, max_frames: int = 12):
+    """Times the oracle on a bounded sample: frames 1.. of the same sequence
+    (selection, readout of every kept row, commit), until the budget is used.
+    Returns (frames timed, seconds, sample description)."""
+    from oracle import oracle as orc
+    from paper_2608_22526_gb300 import synth
+    seq = synth.Sequence(w)
+    ring = w.ring_cap_rows() if w.window > 0 else w.ring_cap_rows_tight()
+    ob = orc.OracleBank(w.U, w.D, w.dtype, w.mn, w.n_cond, w.window, ring, w.max_frames(), w.n_ptr)
+    track = np.zeros((w.U, 6), np.int32)
+    ug = w.unit_group()
+    kn, vn = seq.kv_new(0)
+    m0 = seq.masks(0)
+    if w.n_cond > 0:
+        ob.commit(kn, vn, m0, 1)
+        if w.n_ptr:
+            ob.set_pointers(*seq.pointers())
+    done, spent = 0, 0.0
+    t = 1
+    while t < w.frames and done < max_frames and spent < budget_s:
+        z = seq.z(t)
+        prev = seq.masks(t - 1)
+        kt, vt = seq.kv_new(t)
+        mt = seq.masks(t)
+        x = z[ug].copy()
+        t0 = time.perf_counter()
+        sel = orc.select(z, w.dtype, prev, ug, track, w.m, w.n, w.rho, w.r_s, w.c, w.union_mode)
+        for u in range(w.U):
+            K, V = ob.kv(u)
+            A = orc.readout(z[ug[u]], w.dtype, w.H, w.d, sel.keep(u), K, V, w.dtype,
+                            threads=threads)
+            x[u] = orc.scatter_output(x[u], w.dtype, w.mn, w.D, sel.keep(u), A)
+        ob.commit(kt, vt, mt, 0)
+        spent += time.perf_counter() - t0
+        done += 1
+        t += 1
+    return done, spent, f"frames 1..{done} of {w.name} (select + readout of every kept row + commit), fp64"
+
+
+def cpu_baseline(w, budget_s: float = 15.0):
+    threads = os.cpu_count() or 1
+    n, s, desc = oracle_frames(w, budget_s, threads)
+    return {"value": round(n / s, 4) if s > 0 else None, "unit": "frames/s", "cores": threads,
+            "kind": "oracle", "sample": desc}
+
+
+def reference_arm(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    from paper_2608_22526_gb300 import synth
+    w = synth.WORKLOADS[args.workload]
+    threads = os.cpu_count() or 1
+    # warm-up: one frame each; timed: `steps` frames
+    for _ in range(args.warmup):
+        oracle_frames(w, 1e9, threads, max_frames=1)
+    n, s, desc = oracle_frames(w, 1e9, threads, max_frames=max(1, args.steps))
+    v = n / s if s > 0 else None
+    line = {
+        "metric": METRIC, "value": round(v, 4) if v else None, "unit": "frames/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(s / max(n, 1) * 1e3, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "global_batch": 1, "seq_len": w.frames,
+                   "parallelism": "host cores"},
+        "impl": "reference",
+        "cpu_baseline": {"value": round(v, 4) if v else None, "unit": "frames/s",
+                         "cores": threads, "kind": "oracle", "sample": desc},
+        "e2e": {"value": round(v, 4) if v else None, "unit": "frames/s",
+                "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--no-dense", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    if args.impl == "reference":
+        reference_arm(args)
+    else:
+        gpu_arm(args)
+
+
+if __name__ == "__main__":
+    main()

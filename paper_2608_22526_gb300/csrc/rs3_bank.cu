@@ -1,0 +1,343 @@
+// rs3_bank.cu -- ragged per-unit memory bank and the write-pruned commit
+// (Sec. 3.2, Eq. 8; Algorithm 1's sparse write).
+//
+// A commit is two launches:
+//   k_commit_plan  one CTA per unit: counts the kept rows per 256-cell chunk,
+//                  decides eviction / capacity from the old counters, updates
+//                  the counters and the frame table, and leaves a copy plan.
+//   k_commit_copy  one CTA per (chunk, unit): ballot/popc ranks of the kept
+//                  cells inside the chunk, then warp-per-row 128-bit copies of
+//                  the K and V rows to their bank rows.
+#include "rs3_internal.cuh"
+
+#include <cstdlib>
+#include <cstring>
+
+namespace {
+
+struct BankDev {
+    int64_t *meta;
+    int64_t stride_words;
+    int32_t max_frames, window, n_cond, n_ptr;
+    int64_t pinned_cap, ring_cap, rows_per_unit;
+};
+
+BankDev bank_dev(const rs3_bank *b)
+{
+    BankDev v;
+    v.meta = static_cast<int64_t *>(b->meta);
+    v.stride_words = b->meta_stride / 8;
+    v.max_frames = b->max_frames;
+    v.window = b->window;
+    v.n_cond = b->n_cond;
+    v.n_ptr = b->n_ptr;
+    v.pinned_cap = b->pinned_cap;
+    v.ring_cap = b->ring_cap;
+    v.rows_per_unit = b->rows_per_unit;
+    return v;
+}
+
+__device__ __forceinline__ int32_t *chunk_prefix(int64_t *mu, int max_frames)
+{
+    return reinterpret_cast<int32_t *>(mu + BM_HEADER_WORDS + 2 * (int64_t)max_frames);
+}
+
+__global__ void __launch_bounds__(1024)
+k_commit_plan(const uint8_t *__restrict__ mask, int mn, int is_cond, BankDev bk, int32_t *status)
+{
+    __shared__ int32_t s_cnt[BM_CHUNK_WORDS * 2];
+    const int u = blockIdx.x;
+    int64_t *mu = bk.meta + (int64_t)u * bk.stride_words;
+    const int nchunks = (mn + COMMIT_CHUNK - 1) / COMMIT_CHUNK;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    const uint8_t *Mu = mask ? mask + (size_t)u * mn : nullptr;
+    for (int ch = warp; ch < nchunks; ch += nw) {
+        int c = 0;
+        for (int i = ch * COMMIT_CHUNK + lane; i < min(mn, (ch + 1) * COMMIT_CHUNK); i += 32)
+            c += Mu ? (Mu[i] != 0) : 1;
+        c = warp_sum(c);
+        if (lane == 0) s_cnt[ch] = c;
+    }
+    __syncthreads();
+    if (threadIdx.x != 0) return;
+    int32_t *pref = chunk_prefix(mu, bk.max_frames);
+    int64_t L = 0;
+    for (int ch = 0; ch < nchunks; ++ch) {
+        pref[ch] = (int32_t)L;
+        L += s_cnt[ch];
+    }
+    int64_t *foff = mu + BM_HEADER_WORDS;
+    int64_t *flen = foff + bk.max_frames;
+    bool ok;
+    int64_t base = 0;
+    if (is_cond) {
+        ok = mu[BM_NCOND] < bk.n_cond && mu[BM_COND_LEN] + L <= bk.pinned_cap;
+        if (ok) {
+            base = mu[BM_COND_LEN];
+            mu[BM_COND_LEN] += L;
+            mu[BM_NCOND] += 1;
+        }
+    } else {
+        int64_t head = mu[BM_HEAD], tail = mu[BM_TAIL];
+        int64_t nf = mu[BM_NFRAMES], oldest = mu[BM_OLDEST];
+        if (head < 0 || tail < head || nf < 0 || nf > bk.max_frames || oldest < 0 ||
+            oldest >= bk.max_frames) {
+            latch_status(status, RS3_EINTERNAL);
+            mu[BM_PLAN_OK] = 0;
+            return;
+        }
+        if (bk.window > 0 && nf == bk.window) {      // evict the oldest ring frame
+            head += flen[oldest];
+            oldest = (oldest + 1) % bk.max_frames;
+            nf -= 1;
+        }
+        ok = nf < bk.max_frames && (tail - head) + L <= bk.ring_cap;
+        if (ok) {
+            const int64_t slot = (oldest + nf) % bk.max_frames;
+            foff[slot] = tail;
+            flen[slot] = L;
+            base = tail;
+            mu[BM_HEAD] = head;
+            mu[BM_TAIL] = tail + L;
+            mu[BM_NFRAMES] = nf + 1;
+            mu[BM_OLDEST] = oldest;
+        }
+    }
+    if (!ok) latch_status(status, RS3_ECAPACITY);
+    mu[BM_PLAN_OK] = ok ? 1 : 0;
+    mu[BM_PLAN_COND] = is_cond ? 1 : 0;
+    mu[BM_PLAN_BASE] = base;
+}
+
+// Copies `nvec` 16-byte words of one row (one warp).
+__device__ __forceinline__ void copy_row(uint4 *__restrict__ dk, uint4 *__restrict__ dv,
+                                         const uint4 *__restrict__ sk, const uint4 *__restrict__ sv,
+                                         int nvec, int lane)
+{
+    for (int v = lane; v < nvec; v += 32) {
+        const uint4 a = __ldcs(sk + v);
+        const uint4 b = __ldcs(sv + v);
+        dk[v] = a;
+        dv[v] = b;
+    }
+}
+
+__global__ void __launch_bounds__(256)
+k_commit_copy(const uint8_t *__restrict__ k_new, const uint8_t *__restrict__ v_new,
+              const uint8_t *__restrict__ mask, int mn, int64_t row_bytes, BankDev bk,
+              uint8_t *__restrict__ k_store, uint8_t *__restrict__ v_store)
+{
+    __shared__ int32_t s_list[COMMIT_CHUNK];
+    __shared__ int32_t s_wtot[8];
+    const int u = blockIdx.y, ch = blockIdx.x;
+    const int64_t *mu = bk.meta + (int64_t)u * bk.stride_words;
+    if (mu[BM_PLAN_OK] == 0) return;
+    const bool cond = mu[BM_PLAN_COND] != 0;
+    const int64_t base = mu[BM_PLAN_BASE];
+    const int32_t pre = reinterpret_cast<const int32_t *>(mu + BM_HEADER_WORDS + 2 * (int64_t)bk.max_frames)[ch];
+
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int cell = ch * COMMIT_CHUNK + threadIdx.x;
+    const bool keep = cell < mn && (mask ? mask[(size_t)u * mn + cell] != 0 : true);
+    const uint32_t bal = __ballot_sync(0xffffffffu, keep);
+    if (lane == 0) s_wtot[warp] = __popc(bal);
+    __syncthreads();
+    int off = 0, nk = 0;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) {
+        off += (w < warp) ? s_wtot[w] : 0;
+        nk += s_wtot[w];
+    }
+    if (keep) {
+        uint32_t lm;
+        asm("mov.u32 %0, %%lanemask_lt;" : "=r"(lm));
+        s_list[off + __popc(bal & lm)] = cell;
+    }
+    __syncthreads();
+    const int nvec = (int)(row_bytes / 16);
+    const uint8_t *ksrc = k_new + (size_t)u * mn * row_bytes;
+    const uint8_t *vsrc = v_new + (size_t)u * mn * row_bytes;
+    uint8_t *kdst = k_store + (size_t)u * bk.rows_per_unit * row_bytes;
+    uint8_t *vdst = v_store + (size_t)u * bk.rows_per_unit * row_bytes;
+    for (int j = warp; j < nk; j += 8) {
+        const int64_t rank = (int64_t)pre + j;
+        const int64_t row = cond ? base + rank : bk.pinned_cap + (base + rank) % bk.ring_cap;
+        const int64_t c = s_list[j];
+        copy_row(reinterpret_cast<uint4 *>(kdst + row * row_bytes),
+                 reinterpret_cast<uint4 *>(vdst + row * row_bytes),
+                 reinterpret_cast<const uint4 *>(ksrc + c * row_bytes),
+                 reinterpret_cast<const uint4 *>(vsrc + c * row_bytes), nvec, lane);
+    }
+}
+
+__global__ void k_set_pointers(const uint8_t *__restrict__ kp, const uint8_t *__restrict__ vp,
+                               int64_t row_bytes, BankDev bk, uint8_t *__restrict__ k_store,
+                               uint8_t *__restrict__ v_store)
+{
+    const int u = blockIdx.x;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    const int nvec = (int)(row_bytes / 16);
+    const int64_t row0 = bk.pinned_cap + bk.ring_cap;
+    for (int j = warp; j < bk.n_ptr; j += nw) {
+        const size_t src = ((size_t)u * bk.n_ptr + j) * row_bytes;
+        const size_t dst = ((size_t)u * bk.rows_per_unit + row0 + j) * row_bytes;
+        copy_row(reinterpret_cast<uint4 *>(k_store + dst), reinterpret_cast<uint4 *>(v_store + dst),
+                 reinterpret_cast<const uint4 *>(kp + src), reinterpret_cast<const uint4 *>(vp + src),
+                 nvec, lane);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) bk.meta[(int64_t)u * bk.stride_words + BM_PTRLEN] = bk.n_ptr;
+}
+
+__global__ void k_bank_reset(BankDev bk, int unit, int U)
+{
+    const int u0 = unit < 0 ? 0 : unit, u1 = unit < 0 ? U : unit + 1;
+    for (int u = u0 + blockIdx.x; u < u1; u += gridDim.x) {
+        int64_t *mu = bk.meta + (int64_t)u * bk.stride_words;
+        for (int w = threadIdx.x; w < BM_HEADER_WORDS; w += blockDim.x) mu[w] = 0;
+    }
+}
+
+bool bank_ok(const rs3_bank *b)
+{
+    return b && b->magic == RS3_BANK_MAGIC && b->meta && b->k_store && b->v_store && b->U >= 1;
+}
+
+size_t elem_bytes(int dtype) { return dtype == RS3_BF16 ? 2 : 4; }
+
+}  // namespace
+
+extern "C" rs3_status rs3_bank_layout(int U, int H, int d, rs3_dtype dtype, int mn, int n_cond,
+                                      int window, int64_t ring_cap_rows, int max_frames, int n_ptr,
+                                      int64_t *rows_per_unit, size_t *meta_bytes)
+{
+    if (U < 1 || H < 1 || d < 1 || mn < 1 || n_cond < 0 || n_ptr < 0 || ring_cap_rows < 0)
+        return RS3_EINVAL;
+    if (dtype != RS3_F32 && dtype != RS3_BF16) return RS3_EINVAL;
+    if (mn > RS3_MAX_MN) return RS3_EUNSUPPORTED;
+    if (((int64_t)H * d * (int64_t)elem_bytes(dtype)) % 16 != 0) return RS3_EINVAL;
+    if (window == 0 || window < -1) return RS3_EINVAL;
+    if (window > 0) {
+        if (max_frames != window) return RS3_EINVAL;
+        if (ring_cap_rows < (int64_t)window * mn) return RS3_EINVAL;
+    } else if (max_frames < 1) {
+        return RS3_EINVAL;
+    }
+    const int64_t rows = (int64_t)n_cond * mn + ring_cap_rows + n_ptr;
+    if (rows_per_unit) *rows_per_unit = rows;
+    if (meta_bytes) *meta_bytes = (size_t)U * (size_t)bank_meta_words(max_frames) * 8;
+    return RS3_OK;
+}
+
+extern "C" rs3_status rs3_bank_init(rs3_bank *bank, int U, int H, int d, rs3_dtype dtype, int mn,
+                                    int n_cond, int window, int64_t ring_cap_rows, int max_frames,
+                                    int n_ptr, void *k_store, void *v_store, void *meta,
+                                    rs3_stream_t stream)
+{
+    if (!bank || !k_store || !v_store || !meta) return RS3_EINVAL;
+    int64_t rows;
+    size_t mb;
+    const rs3_status s = rs3_bank_layout(U, H, d, dtype, mn, n_cond, window, ring_cap_rows,
+                                         max_frames, n_ptr, &rows, &mb);
+    if (s != RS3_OK) return s;
+    if (!rs3_aligned16(k_store) || !rs3_aligned16(v_store) || !rs3_aligned16(meta)) return RS3_EINVAL;
+    std::memset(bank, 0, sizeof(*bank));
+    bank->U = U; bank->H = H; bank->d = d; bank->D = H * d;
+    bank->dtype = dtype; bank->mn = mn; bank->n_cond = n_cond; bank->window = window;
+    bank->max_frames = max_frames; bank->n_ptr = n_ptr;
+    bank->pinned_cap = (int64_t)n_cond * mn;
+    bank->ring_cap = ring_cap_rows;
+    bank->rows_per_unit = rows;
+    bank->meta_stride = bank_meta_words(max_frames) * 8;
+    bank->k_store = k_store; bank->v_store = v_store; bank->meta = meta;
+    bank->magic = RS3_BANK_MAGIC;
+    if (cudaMemsetAsync(meta, 0, mb, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return RS3_ECUDA;
+    return RS3_OK;
+}
+
+extern "C" rs3_status rs3_bank_commit(const rs3_bank *bank, const void *k_new, const void *v_new,
+                                      const uint8_t *keep_mask, int is_cond, int32_t *status,
+                                      rs3_stream_t stream)
+{
+    if (!bank_ok(bank) || !k_new || !v_new || !status) return RS3_EINVAL;
+    if (is_cond != 0 && is_cond != 1) return RS3_EINVAL;
+    if (is_cond && bank->n_cond == 0) return RS3_EINVAL;
+    if (!rs3_aligned16(k_new) || !rs3_aligned16(v_new)) return RS3_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const BankDev bk = bank_dev(bank);
+    const int mn = bank->mn;
+    k_commit_plan<<<bank->U, 1024, 0, st>>>(keep_mask, mn, is_cond, bk, status);
+    if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
+    const int nchunks = (mn + COMMIT_CHUNK - 1) / COMMIT_CHUNK;
+    const int64_t row_bytes = (int64_t)bank->D * (int64_t)elem_bytes(bank->dtype);
+    k_commit_copy<<<dim3(nchunks, bank->U), 256, 0, st>>>(
+        static_cast<const uint8_t *>(k_new), static_cast<const uint8_t *>(v_new), keep_mask, mn,
+        row_bytes, bk, static_cast<uint8_t *>(bank->k_store), static_cast<uint8_t *>(bank->v_store));
+    if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
+    return RS3_OK;
+}
+
+extern "C" rs3_status rs3_bank_set_pointers(const rs3_bank *bank, const void *k_ptr,
+                                            const void *v_ptr, int32_t *status, rs3_stream_t stream)
+{
+    if (!bank_ok(bank) || !k_ptr || !v_ptr || !status) return RS3_EINVAL;
+    if (bank->n_ptr == 0) return RS3_EINVAL;
+    if (!rs3_aligned16(k_ptr) || !rs3_aligned16(v_ptr)) return RS3_EINVAL;
+    const int64_t row_bytes = (int64_t)bank->D * (int64_t)elem_bytes(bank->dtype);
+    k_set_pointers<<<bank->U, 256, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+        static_cast<const uint8_t *>(k_ptr), static_cast<const uint8_t *>(v_ptr), row_bytes,
+        bank_dev(bank), static_cast<uint8_t *>(bank->k_store), static_cast<uint8_t *>(bank->v_store));
+    if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
+    return RS3_OK;
+}
+
+extern "C" rs3_status rs3_bank_reset(const rs3_bank *bank, int unit, rs3_stream_t stream)
+{
+    if (!bank_ok(bank)) return RS3_EINVAL;
+    if (unit < -1 || unit >= bank->U) return RS3_EINVAL;
+    const int blocks = unit < 0 ? (bank->U < 1024 ? bank->U : 1024) : 1;
+    k_bank_reset<<<blocks, 32, 0, reinterpret_cast<cudaStream_t>(stream)>>>(bank_dev(bank), unit,
+                                                                            bank->U);
+    if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
+    return RS3_OK;
+}
+
+extern "C" rs3_status rs3_bank_read_meta(const rs3_bank *bank, int64_t *host_out,
+                                         int64_t *frames_out, rs3_stream_t stream)
+{
+    if (!bank_ok(bank) || !host_out) return RS3_EINVAL;
+    const size_t words = (size_t)bank->U * (size_t)(bank->meta_stride / 8);
+    int64_t *tmp = static_cast<int64_t *>(std::malloc(words * 8));
+    if (!tmp) return RS3_ECAPACITY;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(tmp, bank->meta, words * 8, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess) {
+        std::free(tmp);
+        return RS3_ECUDA;
+    }
+    const int64_t sw = bank->meta_stride / 8;
+    for (int u = 0; u < bank->U; ++u) {
+        const int64_t *mu = tmp + u * sw;
+        int64_t *o = host_out + 8 * (int64_t)u;
+        for (int w = 0; w < 7; ++w) o[w] = mu[w];
+        o[7] = mu[BM_COND_LEN] + (mu[BM_TAIL] - mu[BM_HEAD]) + mu[BM_PTRLEN];
+        if (frames_out) {
+            const int64_t *foff = mu + BM_HEADER_WORDS;
+            const int64_t *flen = foff + bank->max_frames;
+            int64_t *fo = frames_out + (int64_t)u * bank->max_frames * 2;
+            for (int i = 0; i < bank->max_frames; ++i) {
+                if (i < mu[BM_NFRAMES]) {
+                    const int64_t s = (mu[BM_OLDEST] + i) % bank->max_frames;
+                    fo[2 * i] = foff[s];
+                    fo[2 * i + 1] = flen[s];
+                } else {
+                    fo[2 * i] = -1;
+                    fo[2 * i + 1] = -1;
+                }
+            }
+        }
+    }
+    std::free(tmp);
+    return RS3_OK;
+}

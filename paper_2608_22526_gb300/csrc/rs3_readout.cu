@@ -1,0 +1,580 @@
+// rs3_readout.cu -- pruned memory readout (Sec. 3.1: Eq. 6 gather / attention /
+// scatter, Eq. 7 RoPE by the gathered index), host entry and the shared
+// pieces of both kernel paths.
+//
+// Launch sequence (one stream, no host synchronisation):
+//   k_passthrough  out-of-place only: out = residual (or zeros) on every cell
+//   k_plan         one CTA: per unit, the bank's row ranges (pinned, ring
+//                  pieces, pointers) and a balanced work list of
+//                  (unit, head, query tile, KV tile range) items; long banks
+//                  are split along the keys so every SM gets work
+//   k_readout_*    flash attention per item: gather the kept query rows (and
+//                  rotate them), stream the bank tiles, online softmax in the
+//                  log2 domain, fp32 accumulation; an unsplit item writes
+//                  out = residual + A directly at the kept cells, a split item
+//                  writes (O, m, l) partials
+//   k_combine      log-sum-exp merge of the partials and the scatter
+#include "rs3_internal.cuh"
+
+#include <cmath>
+
+#include "rs3_readout_common.cuh"
+
+namespace {
+
+// ---------------------------------------------------------------------------
+// k_passthrough: unselected cells equal the residual bit for bit (Eq. 6 S_K)
+// ---------------------------------------------------------------------------
+__global__ void k_passthrough(const uint4 *__restrict__ res, uint4 *__restrict__ out, int64_t nvec)
+{
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nvec;
+         i += (int64_t)gridDim.x * blockDim.x)
+        out[i] = res ? __ldcs(res + i) : make_uint4(0, 0, 0, 0);
+}
+
+// ---------------------------------------------------------------------------
+// k_plan: ranges and the work list
+// ---------------------------------------------------------------------------
+__device__ RangeSet unit_ranges(const ReadoutArgs &a, int u, int cnt)
+{
+    RangeSet rs;
+    const int64_t *mu = a.meta + (int64_t)u * a.meta_stride_words;
+    const int64_t cond = mu[BM_COND_LEN];
+    const int64_t head = mu[BM_HEAD], tail = mu[BM_TAIL], ptr = mu[BM_PTRLEN];
+    for (int r = 0; r < 4; ++r) { rs.start[r] = 0; rs.len[r] = 0; rs.tiles[r] = 0; }
+    rs.start[0] = 0;
+    rs.len[0] = (int32_t)cond;
+    const int64_t live = tail - head;
+    if (live > 0 && a.ring_cap > 0) {
+        const int64_t p0 = head % a.ring_cap;
+        const int64_t first = min(live, a.ring_cap - p0);
+        rs.start[1] = a.pinned_cap + p0;
+        rs.len[1] = (int32_t)first;
+        rs.start[2] = a.pinned_cap;
+        rs.len[2] = (int32_t)(live - first);
+    }
+    rs.start[3] = a.pinned_cap + a.ring_cap;
+    rs.len[3] = (int32_t)ptr;
+    int nt = 0;
+    for (int r = 0; r < 4; ++r) {
+        rs.tiles[r] = (rs.len[r] + a.BN - 1) / a.BN;
+        nt += rs.tiles[r];
+    }
+    rs.n_tiles = nt;
+    rs.cnt = cnt;
+    rs.nq = (cnt + a.BM - 1) / a.BM;
+    rs.splits = 1;
+    rs.slot_base = -1;
+    return rs;
+}
+
+__device__ __forceinline__ int splits_for(int n_tiles, int64_t chunk)
+{
+    if (n_tiles <= 1) return 1;
+    int64_t s = (n_tiles + chunk - 1) / chunk;
+    if (s > RS3_MAX_SPLITS) s = RS3_MAX_SPLITS;
+    if (s > n_tiles) s = n_tiles;
+    return s < 1 ? 1 : (int)s;
+}
+
+__device__ int64_t block_sum64(int64_t v)
+{
+    __shared__ int64_t s_part[32];
+    __shared__ int64_t s_tot;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (lane == 0) s_part[warp] = v;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int64_t t = 0;
+        for (int w = 0; w < nw; ++w) t += s_part[w];
+        s_tot = t;
+    }
+    __syncthreads();
+    const int64_t r = s_tot;
+    __syncthreads();
+    return r;
+}
+
+// exclusive scan of an int64 per thread, returns offset; *total = block total
+__device__ int64_t block_scan64(int64_t v, int64_t *total)
+{
+    __shared__ int64_t s_part[32];
+    __shared__ int64_t s_tot;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    int64_t incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int64_t t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += t;
+    }
+    if (lane == 31) s_part[warp] = incl;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int64_t run = 0;
+        for (int w = 0; w < nw; ++w) {
+            const int64_t t = s_part[w];
+            s_part[w] = run;
+            run += t;
+        }
+        s_tot = run;
+    }
+    __syncthreads();
+    const int64_t off = s_part[warp] + incl - v;
+    *total = s_tot;
+    __syncthreads();
+    return off;
+}
+
+__global__ void __launch_bounds__(1024) k_plan(ReadoutArgs a)
+{
+    ReadoutHeader *hdr = a.header;
+    int64_t work_local = 0;
+    for (int u = threadIdx.x; u < a.U; u += blockDim.x) {
+        int cnt = a.count[u];
+        if (cnt < 0 || cnt > a.k_max) {
+            latch_status(a.status, RS3_EINVAL);
+            cnt = cnt < 0 ? 0 : a.k_max;
+        }
+        const int64_t *mu = a.meta + (int64_t)u * a.meta_stride_words;
+        const bool sane = mu[BM_HEAD] >= 0 && mu[BM_TAIL] >= mu[BM_HEAD] &&
+                          mu[BM_TAIL] - mu[BM_HEAD] <= a.ring_cap && mu[BM_COND_LEN] >= 0 &&
+                          mu[BM_COND_LEN] <= a.pinned_cap && mu[BM_PTRLEN] >= 0 &&
+                          mu[BM_PTRLEN] <= a.n_ptr;
+        RangeSet rs;
+        if (!sane) {
+            latch_status(a.status, RS3_EINTERNAL);
+            for (int r = 0; r < 4; ++r) { rs.start[r] = 0; rs.len[r] = 0; rs.tiles[r] = 0; }
+            rs.n_tiles = 0; rs.cnt = 0; rs.nq = 0; rs.splits = 1; rs.slot_base = -1;
+        } else {
+            rs = unit_ranges(a, u, cnt);
+        }
+        a.ranges[u] = rs;
+        work_local += (int64_t)rs.nq * a.H * (rs.n_tiles > 0 ? rs.n_tiles : 1);
+    }
+    const int64_t W = block_sum64(work_local);     // syncs: ranges visible
+    int64_t chunk = (W + a.n_sm - 1) / a.n_sm;
+    if (chunk < a.min_chunk) chunk = a.min_chunk;
+    for (int iter = 0; iter < 40; ++iter) {
+        int64_t slots_local = 0;
+        for (int u = threadIdx.x; u < a.U; u += blockDim.x) {
+            const RangeSet &rs = a.ranges[u];
+            const int s = splits_for(rs.n_tiles, chunk);
+            if (s > 1) slots_local += (int64_t)rs.nq * a.H * s;
+        }
+        const int64_t S = block_sum64(slots_local);
+        if (S <= a.max_slots) break;
+        chunk *= 2;
+    }
+    // offsets, rounds of blockDim units
+    int64_t item_run = 0, slot_run = 0, comb_run = 0;
+    for (int u0 = 0; u0 < a.U; u0 += blockDim.x) {
+        const int u = u0 + threadIdx.x;
+        int64_t ni = 0, ns = 0, nc = 0;
+        int s = 1;
+        if (u < a.U) {
+            s = splits_for(a.ranges[u].n_tiles, chunk);
+            ni = (int64_t)a.ranges[u].nq * a.H * s;
+            ns = s > 1 ? ni : 0;
+            nc = s > 1 ? (int64_t)a.ranges[u].nq * a.H : 0;
+        }
+        int64_t ti, ts, tc;
+        const int64_t oi = block_scan64(ni, &ti) + item_run;
+        const int64_t os = block_scan64(ns, &ts) + slot_run;
+        const int64_t oc = block_scan64(nc, &tc) + comb_run;
+        if (u < a.U) {
+            RangeSet rs = a.ranges[u];
+            rs.splits = s;
+            rs.slot_base = s > 1 ? (int32_t)os : -1;
+            a.ranges[u] = rs;
+            int64_t it = oi, ic = oc;
+            for (int qt = 0; qt < rs.nq; ++qt)
+                for (int h = 0; h < a.H; ++h) {
+                    const int32_t slot0 = s > 1 ? (int32_t)(os + ((int64_t)qt * a.H + h) * s) : -1;
+                    for (int sp = 0; sp < s; ++sp) {
+                        WorkItem w;
+                        w.u = u; w.h = h; w.qt = qt; w.split = sp;
+                        w.tile_begin = (int32_t)((int64_t)sp * rs.n_tiles / s);
+                        w.tile_end = (int32_t)((int64_t)(sp + 1) * rs.n_tiles / s);
+                        w.slot = s > 1 ? slot0 + sp : -1;
+                        w.pad = 0;
+                        a.items[it++] = w;
+                    }
+                    if (s > 1) {
+                        CombineItem c;
+                        c.u = u; c.h = h; c.qt = qt; c.slot0 = slot0; c.nsplit = s;
+                        c.pad[0] = c.pad[1] = c.pad[2] = 0;
+                        a.combine[ic++] = c;
+                    }
+                }
+        }
+        item_run += ti;
+        slot_run += ts;
+        comb_run += tc;
+    }
+    if (threadIdx.x == 0) {
+        hdr->n_items = (int32_t)item_run;
+        hdr->n_combine = (int32_t)comb_run;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// k_readout_simt: CUDA-core flash readout (fp32 path; any dtype)
+// ---------------------------------------------------------------------------
+// One CTA per work item of BM = 32 query rows.  A row is owned by TPR = d/16
+// threads, each holding 16 dimensions of q~ and of the output accumulator.
+// Keys are staged 32 at a time in shared memory as fp32.
+constexpr int SIMT_BM = 32;
+constexpr int SIMT_BN = 32;
+
+template <typename T>
+__global__ void __launch_bounds__(512) k_readout_simt(ReadoutArgs a)
+{
+    extern __shared__ __align__(16) float sm[];
+    const int d = a.d;
+    const int TPR = d / 16;
+    float *sK = sm;                      // [SIMT_BN][d]
+    float *sV = sm + SIMT_BN * d;        // [SIMT_BN][d]
+    const int n_items = a.header->n_items;
+    for (int it = blockIdx.x; it < n_items; it += gridDim.x) {
+        const WorkItem w = a.items[it];
+        const RangeSet rs = a.ranges[w.u];
+        const int r = threadIdx.x / TPR;
+        const int part = threadIdx.x % TPR;
+        const int j = w.qt * SIMT_BM + r;
+        const bool valid = j < rs.cnt;
+        const int g = a.unit_group[w.u];
+        if (g < 0 || g >= a.G) {                 // uniform over the CTA
+            if (threadIdx.x == 0) latch_status(a.status, RS3_EINVAL);
+            continue;
+        }
+        int cell = 0;
+        if (valid) cell = a.idx[(int64_t)w.u * a.k_max + j];
+        if (cell < 0 || cell >= a.mn) cell = 0;
+        const int c0 = w.h * d + part * 16;
+        float qv[16];
+        {
+            const T *qr = static_cast<const T *>(a.q) + ((int64_t)g * a.mn + cell) * a.D + c0;
+            load16(qr, qv);
+            if (a.rope) {
+                const float *f = a.rope + ((int64_t)cell * (d / 2) + part * 8) * 2;
+#pragma unroll
+                for (int p = 0; p < 8; ++p) {
+                    const float cs = f[2 * p], sn = f[2 * p + 1];
+                    const float x0 = qv[2 * p], x1 = qv[2 * p + 1];
+                    qv[2 * p] = x0 * cs - x1 * sn;
+                    qv[2 * p + 1] = x0 * sn + x1 * cs;
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < 16; ++k) qv[k] *= a.scale_log2;
+        }
+        float o[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) o[k] = 0.f;
+        float mrun = -INFINITY, lrun = 0.f;
+        const T *Kb = static_cast<const T *>(a.k_store) + (int64_t)w.u * a.rows_per_unit * a.D;
+        const T *Vb = static_cast<const T *>(a.v_store) + (int64_t)w.u * a.rows_per_unit * a.D;
+        for (int t = w.tile_begin; t < w.tile_end; ++t) {
+            int64_t row0;
+            int nvalid;
+            tile_rows(rs, t, SIMT_BN, row0, nvalid);
+            if (nvalid <= 0) continue;           // uniform over the CTA
+            __syncthreads();
+            // stage keys / values of this head as fp32
+            const int vec_per_row = d / 4;
+            for (int e = threadIdx.x; e < SIMT_BN * vec_per_row; e += blockDim.x) {
+                const int kk = e / vec_per_row, c4 = (e % vec_per_row) * 4;
+                float4 kv = make_float4(0.f, 0.f, 0.f, 0.f), vv = kv;
+                if (kk < nvalid) {
+                    kv = load4(Kb + (row0 + kk) * a.D + w.h * d + c4);
+                    vv = load4(Vb + (row0 + kk) * a.D + w.h * d + c4);
+                }
+                *reinterpret_cast<float4 *>(sK + kk * d + c4) = kv;
+                *reinterpret_cast<float4 *>(sV + kk * d + c4) = vv;
+            }
+            __syncthreads();
+            float s[SIMT_BN];
+#pragma unroll
+            for (int kk = 0; kk < SIMT_BN; ++kk) {
+                const float *kr = sK + kk * d + part * 16;
+                float acc = 0.f;
+#pragma unroll
+                for (int k = 0; k < 16; ++k) acc = fmaf(qv[k], kr[k], acc);
+                s[kk] = acc;
+            }
+            for (int off = TPR >> 1; off >= 1; off >>= 1) {
+#pragma unroll
+                for (int kk = 0; kk < SIMT_BN; ++kk) s[kk] += __shfl_xor_sync(0xffffffffu, s[kk], off);
+            }
+            float mt = -INFINITY;
+#pragma unroll
+            for (int kk = 0; kk < SIMT_BN; ++kk) {
+                if (kk >= nvalid) s[kk] = -INFINITY;
+                mt = fmaxf(mt, s[kk]);
+            }
+            const float mnew = fmaxf(mrun, mt);
+            const float alpha = exp2f(mrun - mnew);
+            lrun *= alpha;
+#pragma unroll
+            for (int k = 0; k < 16; ++k) o[k] *= alpha;
+#pragma unroll
+            for (int kk = 0; kk < SIMT_BN; ++kk) {
+                const float p = exp2f(s[kk] - mnew);
+                lrun += p;
+                const float *vr = sV + kk * d + part * 16;
+#pragma unroll
+                for (int k = 0; k < 16; ++k) o[k] = fmaf(p, vr[k], o[k]);
+            }
+            mrun = mnew;
+        }
+        if (valid) {
+            if (w.slot < 0) {
+                const float inv = lrun > 0.f ? 1.f / lrun : 0.f;
+#pragma unroll
+                for (int k = 0; k < 16; ++k) o[k] *= inv;
+                store_out16<T>(a, w.u, cell, c0, o);
+            } else {
+                float *po = a.part_o + ((int64_t)w.slot * a.BM + r) * d + part * 16;
+#pragma unroll
+                for (int k = 0; k < 16; k += 4)
+                    *reinterpret_cast<float4 *>(po + k) = make_float4(o[k], o[k + 1], o[k + 2], o[k + 3]);
+                if (part == 0) {
+                    float2 *pm = reinterpret_cast<float2 *>(a.part_ml) + (int64_t)w.slot * a.BM + r;
+                    *pm = make_float2(mrun, lrun);
+                }
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// k_combine: log-sum-exp merge of split-KV partials, then the scatter
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) k_combine(ReadoutArgs a)
+{
+    const int n_comb = a.header->n_combine;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    const int d = a.d;
+    for (int ci = blockIdx.x; ci < n_comb; ci += gridDim.x) {
+        const CombineItem c = a.combine[ci];
+        const RangeSet rs = a.ranges[c.u];
+        const int rows = min(a.BM, rs.cnt - c.qt * a.BM);
+        for (int r = warp; r < rows; r += nw) {
+            const int j = c.qt * a.BM + r;
+            int cell = a.idx[(int64_t)c.u * a.k_max + j];
+            if (cell < 0 || cell >= a.mn) cell = 0;
+            const float2 *pm = reinterpret_cast<const float2 *>(a.part_ml);
+            float M = -INFINITY;
+            for (int s = 0; s < c.nsplit; ++s) M = fmaxf(M, pm[(int64_t)(c.slot0 + s) * a.BM + r].x);
+            float L = 0.f;
+            for (int s = 0; s < c.nsplit; ++s) {
+                const float2 ml = pm[(int64_t)(c.slot0 + s) * a.BM + r];
+                L += (M == -INFINITY) ? 0.f : exp2f(ml.x - M) * ml.y;
+            }
+            const float inv = L > 0.f ? 1.f / L : 0.f;
+            for (int c4 = lane * 4; c4 < d; c4 += 128) {
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int s = 0; s < c.nsplit; ++s) {
+                    const float2 ml = pm[(int64_t)(c.slot0 + s) * a.BM + r];
+                    const float wgt = (M == -INFINITY) ? 0.f : exp2f(ml.x - M);
+                    const float4 po = *reinterpret_cast<const float4 *>(
+                        a.part_o + ((int64_t)(c.slot0 + s) * a.BM + r) * d + c4);
+                    acc.x = fmaf(wgt, po.x, acc.x);
+                    acc.y = fmaf(wgt, po.y, acc.y);
+                    acc.z = fmaf(wgt, po.z, acc.z);
+                    acc.w = fmaf(wgt, po.w, acc.w);
+                }
+                float o4[4] = {acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv};
+                store_out4<T>(a, c.u, cell, c.h * d + c4, o4);
+            }
+        }
+    }
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+namespace {
+
+ReadoutLayout readout_layout(int U, int H, int d, int k_max, int BM)
+{
+    ReadoutLayout L;
+    const int64_t nq = k_max > 0 ? (k_max + BM - 1) / BM : 1;
+    L.max_slots = RS3_MAX_SLOTS;
+    L.max_combine = (int64_t)U * H * nq;
+    L.max_items = L.max_combine + L.max_slots;
+    size_t off = 0;
+    L.header = off;
+    off = align_up(off + sizeof(ReadoutHeader), 256);
+    L.ranges = off;
+    off = align_up(off + (size_t)U * sizeof(RangeSet), 256);
+    L.items = off;
+    off = align_up(off + (size_t)L.max_items * sizeof(WorkItem), 256);
+    L.combine = off;
+    off = align_up(off + (size_t)L.max_combine * sizeof(CombineItem), 256);
+    L.part_o = off;
+    off = align_up(off + (size_t)L.max_slots * BM * d * 4, 256);
+    L.part_ml = off;
+    off = align_up(off + (size_t)L.max_slots * BM * 8, 256);
+    L.total = off;
+    return L;
+}
+
+}  // namespace
+
+ReadoutPath choose_readout_path(rs3_dtype dtype, int d)
+{
+    ReadoutPath p;
+    if (dtype == RS3_BF16 && rs3_tc_supported(d)) {
+        p.kind = 1;
+        p.BM = 128;
+        p.BN = rs3_tc_block_n(d);
+    } else {
+        p.kind = 0;
+        p.BM = SIMT_BM;
+        p.BN = SIMT_BN;
+    }
+    return p;
+}
+
+extern "C" size_t rs3_readout_workspace_bytes(int U, int H, int d, int k_max, rs3_dtype dtype)
+{
+    if (U < 1 || H < 1 || d < 1 || k_max < 0) return 0;
+    const ReadoutPath p = choose_readout_path(dtype, d);
+    return readout_layout(U, H, d, k_max, p.BM).total;
+}
+
+rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, int H, int d,
+                               const int32_t *unit_group, const int32_t *idx, const int32_t *count,
+                               int k_max, const rs3_bank *bank, const float *rope,
+                               const void *residual, void *out, float scale, void *workspace,
+                               size_t workspace_bytes, int32_t *status, ReadoutArgs *a,
+                               ReadoutPath *path, int64_t *grid_items, int64_t *grid_combine)
+{
+    if (!q || !unit_group || !idx || !count || !bank || !out || !workspace || !status)
+        return RS3_EINVAL;
+    if (bank->magic != RS3_BANK_MAGIC || !bank->meta || !bank->k_store || !bank->v_store)
+        return RS3_EINVAL;
+    if (dtype != RS3_F32 && dtype != RS3_BF16) return RS3_EINVAL;
+    if ((int)dtype != bank->dtype || H != bank->H || d != bank->d) return RS3_EINVAL;
+    if (G < 1 || mn < 1 || H < 1 || d < 1 || k_max < 0) return RS3_EINVAL;
+    if (mn > RS3_MAX_MN) return RS3_EUNSUPPORTED;
+    if (d < 16 || d > 256 || (d & (d - 1)) != 0) return RS3_EUNSUPPORTED;
+    if (!rs3_aligned16(q) || !rs3_aligned16(out) || !rs3_aligned16(workspace) ||
+        (residual && !rs3_aligned16(residual)) || (rope && !rs3_aligned16(rope)))
+        return RS3_EINVAL;
+    const ReadoutPath p = choose_readout_path(dtype, d);
+    const ReadoutLayout L = readout_layout(bank->U, H, d, k_max, p.BM);
+    if (workspace_bytes < L.total) return RS3_ECAPACITY;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    a->q = q;
+    a->k_store = bank->k_store;
+    a->v_store = bank->v_store;
+    a->meta = static_cast<const int64_t *>(bank->meta);
+    a->meta_stride_words = bank->meta_stride / 8;
+    a->pinned_cap = bank->pinned_cap;
+    a->ring_cap = bank->ring_cap;
+    a->rows_per_unit = bank->rows_per_unit;
+    a->n_ptr = bank->n_ptr;
+    a->unit_group = unit_group;
+    a->idx = idx;
+    a->count = count;
+    a->rope = rope;
+    a->residual = residual;
+    a->out = out;
+    a->status = status;
+    a->U = bank->U;
+    a->G = G;
+    a->mn = mn;
+    a->H = H;
+    a->d = d;
+    a->D = H * d;
+    a->k_max = k_max;
+    a->BM = p.BM;
+    a->BN = p.BN;
+    a->n_sm = rs3_sm_count();
+    a->min_chunk = p.kind == 1 ? 2 : 4;
+    a->max_slots = L.max_slots;
+    const float sc = scale > 0.f ? scale : 1.0f / sqrtf((float)d);
+    a->scale_log2 = sc * 1.4426950408889634f;
+    a->header = reinterpret_cast<ReadoutHeader *>(ws + L.header);
+    a->ranges = reinterpret_cast<RangeSet *>(ws + L.ranges);
+    a->items = reinterpret_cast<WorkItem *>(ws + L.items);
+    a->combine = reinterpret_cast<CombineItem *>(ws + L.combine);
+    a->part_o = reinterpret_cast<float *>(ws + L.part_o);
+    a->part_ml = reinterpret_cast<float *>(ws + L.part_ml);
+    *path = p;
+    *grid_items = L.max_items;
+    *grid_combine = L.max_combine;
+    return RS3_OK;
+}
+
+rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_t max_items,
+                              int64_t max_combine, rs3_dtype dtype, cudaStream_t st)
+{
+    if (a.residual != a.out) {
+        const int64_t nvec = (int64_t)a.U * a.mn * a.D * (dtype == RS3_BF16 ? 2 : 4) / 16;
+        int64_t blocks = (nvec + 255) / 256;
+        const int64_t cap = (int64_t)a.n_sm * 8;
+        if (blocks > cap) blocks = cap;
+        k_passthrough<<<(unsigned)blocks, 256, 0, st>>>(static_cast<const uint4 *>(a.residual),
+                                                        static_cast<uint4 *>(a.out), nvec);
+        if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
+    }
+    k_plan<<<1, 1024, 0, st>>>(a);
+    if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
+    if (p.kind == 1) {
+        const rs3_status s = rs3_launch_tc_readout(a, st);
+        if (s != RS3_OK) return s;
+    } else {
+        const size_t smem = (size_t)2 * SIMT_BN * a.d * sizeof(float);
+        const int threads = 2 * a.d;
+        int64_t blocks = max_items;
+        const int64_t cap = (int64_t)a.n_sm * 16;
+        if (blocks > cap) blocks = cap;
+        static bool attr_done = false;
+        if (!attr_done) {
+            const int most = 2 * SIMT_BN * 256 * (int)sizeof(float);
+            cudaFuncSetAttribute(k_readout_simt<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+            cudaFuncSetAttribute(k_readout_simt<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+            attr_done = true;
+        }
+        if (dtype == RS3_BF16)
+            k_readout_simt<uint16_t><<<(unsigned)blocks, threads, smem, st>>>(a);
+        else
+            k_readout_simt<float><<<(unsigned)blocks, threads, smem, st>>>(a);
+        if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
+    }
+    int64_t cblocks = max_combine;
+    const int64_t ccap = (int64_t)a.n_sm * 8;
+    if (cblocks > ccap) cblocks = ccap;
+    if (cblocks < 1) cblocks = 1;
+    if (dtype == RS3_BF16)
+        k_combine<uint16_t><<<(unsigned)cblocks, 256, 0, st>>>(a);
+    else
+        k_combine<float><<<(unsigned)cblocks, 256, 0, st>>>(a);
+    if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
+    return RS3_OK;
+}
+
+extern "C" rs3_status rs3_memory_readout(const void *q, rs3_dtype dtype, int G, int mn, int H,
+                                         int d, const int32_t *unit_group, const int32_t *idx,
+                                         const int32_t *count, int k_max, const rs3_bank *bank,
+                                         const float *rope, const void *residual, void *out,
+                                         float scale, void *workspace, size_t workspace_bytes,
+                                         int32_t *status, rs3_stream_t stream)
+{
+    ReadoutArgs a;
+    ReadoutPath p;
+    int64_t gi, gc;
+    const rs3_status s = rs3_readout_prepare(q, dtype, G, mn, H, d, unit_group, idx, count, k_max,
+                                             bank, rope, residual, out, scale, workspace,
+                                             workspace_bytes, status, &a, &p, &gi, &gc);
+    if (s != RS3_OK) return s;
+    return rs3_readout_launch(a, p, gi, gc, dtype, reinterpret_cast<cudaStream_t>(stream));
+}

@@ -12,8 +12,8 @@ Stand-ins (the paper's datasets and checkpoints are not available):
   * queries q_t = Z_t (identity projection);
   * memory-encoder output K_t, V_t [mn, D] per unit: N(0,1);
   * per-object masks at grid resolution: filled ellipses whose centre drifts
-    with a bounded velocity (reflecting at the borders) and whose area follows a
-    bounded random walk inside the configured coverage range;
+    with a bounded velocity (reflecting at the borders) and whose area sweeps
+    the configured coverage range along the sequence;
   * RoPE table f [mn, d/2] as (cos, sin), 2-D axial frequencies (Sec. 3.1, Eq. 7
     uses a table indexed by grid position).
 
@@ -121,7 +121,7 @@ class Workload:
 
 WORKLOADS = {
     # tiny single step, fp32: 32x32 grid, 1 head x 64; bank = 2 unpruned frames
-    "tiny_fp32": Workload("tiny_fp32", 1, 32, 32, 1, 64, "f32", 1, 1, 2,
+    "tiny_fp32": Workload("tiny_fp32", 1, 32, 32, 1, 64, "f32", 1, 1, 1,
                           0.08, 0.12, 0, -1, 0, prefill_frames=2),
     # SAM2-shaped single object, bf16: 64x64, 1 head x 256, cond + 6 recent
     # frames write-pruned to their masks + 16 pointer rows, 60 frames
@@ -190,26 +190,29 @@ class Trajectory:
 def make_trajectory(rng: np.random.Generator, m: int, n: int, frames: int,
                     cov_lo: float, cov_hi: float,
                     vanish: Optional[List[range]] = None) -> Trajectory:
-    """Drifting ellipse: |velocity| <= 1.5 cells/frame, reflecting at the
-    borders; coverage follows a bounded random walk in [cov_lo, cov_hi]."""
+    """Drifting ellipse: |velocity| <= 1.5 cells/frame, reflecting so that the
+    ellipse stays on the grid; its coverage sweeps [cov_lo, cov_hi] along the
+    sequence (a sinusoid of random phase and a period near the length)."""
     mn = m * n
-    cov = rng.uniform(cov_lo, cov_hi)
+    # coverage sweeps the configured range along the sequence (random phase)
+    phase = rng.uniform(0.0, 2 * math.pi)
+    period = rng.uniform(0.8, 1.2) * max(30, frames)
     aspect = rng.uniform(0.6, 1.6)
     theta = rng.uniform(0.0, math.pi)
     speed = rng.uniform(0.3, 1.5)
     ang = rng.uniform(0.0, 2 * math.pi)
     vy, vx = speed * math.sin(ang), speed * math.cos(ang)
-    cy = rng.uniform(0.3 * m, 0.7 * m)
-    cx = rng.uniform(0.3 * n, 0.7 * n)
+    cy = rng.uniform(0.4 * m, 0.6 * m)
+    cx = rng.uniform(0.4 * n, 0.6 * n)
     out = {k: np.zeros(frames) for k in ("cy", "cx", "a", "b", "theta")}
     for t in range(frames):
+        cov = cov_lo + (cov_hi - cov_lo) * 0.5 * (1.0 + math.sin(phase + 2 * math.pi * t / period))
         area = cov * mn
         a = math.sqrt(area * aspect / math.pi)
         b = math.sqrt(area / (aspect * math.pi))
         out["cy"][t], out["cx"][t] = cy, cx
         out["a"][t], out["b"][t], out["theta"][t] = a, b, theta
         # advance
-        cov = min(cov_hi, max(cov_lo, cov + rng.normal(0.0, 0.01 * (cov_hi - cov_lo) + 0.002)))
         theta += rng.normal(0.0, 0.05)
         vy += rng.normal(0.0, 0.15)
         vx += rng.normal(0.0, 0.15)
@@ -218,12 +221,19 @@ def make_trajectory(rng: np.random.Generator, m: int, n: int, frames: int,
             vy, vx = vy * 1.5 / sp, vx * 1.5 / sp
         cy += vy
         cx += vx
-        if cy < 0.0 or cy > m:
+        # keep the whole ellipse on the grid (half-extents of the rotated
+        # ellipse's bounding box), reflecting the velocity at the borders
+        ct, st = math.cos(theta), math.sin(theta)
+        hx = math.sqrt((a * ct) ** 2 + (b * st) ** 2)
+        hy = math.sqrt((a * st) ** 2 + (b * ct) ** 2)
+        lo_y, hi_y = min(hy, m / 2.0), max(m - hy, m / 2.0)
+        lo_x, hi_x = min(hx, n / 2.0), max(n - hx, n / 2.0)
+        if cy < lo_y or cy > hi_y:
             vy = -vy
-            cy = min(float(m), max(0.0, cy))
-        if cx < 0.0 or cx > n:
+            cy = min(hi_y, max(lo_y, cy))
+        if cx < lo_x or cx > hi_x:
             vx = -vx
-            cx = min(float(n), max(0.0, cx))
+            cx = min(hi_x, max(lo_x, cx))
     visible = np.ones(frames, dtype=bool)
     for r in vanish or []:
         for t in r:
