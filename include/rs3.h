@@ -144,6 +144,33 @@ rs3_status rs3_select_queries(const void *z, rs3_dtype dtype, int G, int m, int 
                               int32_t *count, void *workspace, size_t workspace_bytes,
                               int32_t *status, rs3_stream_t stream);
 
+/*
+ * rs3_select_queries for callers that cannot allocate device memory.  The
+ * paper has no counterpart: this is a deployment convenience of the library.
+ * Some callers have no allocator to ask for the workspace (code running while
+ * a stream is captured in the global capture mode, serving loops that must not
+ * allocate after start-up, hosts that pass only input and output buffers
+ * through a plugin interface); this call instead uses scratch memory compiled
+ * into the library: an 8 MiB device array that every GPU loading the library
+ * holds until the process exits.  Arguments and results are those of
+ * rs3_select_queries without the workspace pair.
+ *   - Sizes whose workspace (rs3_select_workspace_bytes(G, U, m, n)) exceeds
+ *     8 MiB are rejected with RS3_ECAPACITY; nothing is launched.
+ *   - The call allocates nothing (no cudaMalloc / cudaFree, no allocating
+ *     library routine).
+ *   - The first call on a device looks up the array's device address with
+ *     that device current and caches it; make that first call before any
+ *     stream capture.
+ *   - All calls on a device share the one array, and it keeps the previous
+ *     call's contents (the call clears what must start at zero itself), so
+ *     calls whose executions overlap on the GPU (different streams without
+ *     ordering between them) race and must not be issued.
+ */
+rs3_status rs3_select_queries_noalloc(const void *z, rs3_dtype dtype, int G, int m, int n, int C,
+                                      const uint8_t *prev_masks, const int32_t *unit_group, int U,
+                                      rs3_track *track, const rs3_params *p, int32_t *idx,
+                                      int32_t *count, int32_t *status, rs3_stream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* Memory bank (Sec. 3.2; Algorithm 1's sparse write)                        */
 /* ------------------------------------------------------------------------ */

@@ -58,6 +58,7 @@ SIGNATURES = {
     "rs3_version": (_I, []),
     "rs3_select_workspace_bytes": (_SZ, [_I, _I, _I, _I]),
     "rs3_select_queries": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _I, _P, _P, _P, _P, _P, _SZ, _P, _P]),
+    "rs3_select_queries_noalloc": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _I, _P, _P, _P, _P, _P, _P]),
     "rs3_bank_layout": (_I, [_I, _I, _I, _I, _I, _I, _I, _I64, _I, _I, _P, _P]),
     "rs3_bank_init": (_I, [_P, _I, _I, _I, _I, _I, _I, _I, _I64, _I, _I, _P, _P, _P, _P]),
     "rs3_bank_commit": (_I, [_P, _P, _P, _P, _I, _P, _P]),
@@ -143,6 +144,16 @@ def rs3_select_queries(z, dtype: str, G: int, m: int, n: int, C: int, prev_masks
                                 _ptr(count), _ptr(workspace), workspace.numel() * workspace.element_size(),
                                 _ptr(status), _stream(stream))
     _check(rc, "rs3_select_queries")
+
+
+def rs3_select_queries_noalloc(z, dtype: str, G: int, m: int, n: int, C: int, prev_masks,
+                               unit_group, U: int, track, params: Params, idx, count, status,
+                               stream=None):
+    """rs3_select_queries with the library's built-in scratch (no workspace)."""
+    rc = lib.rs3_select_queries_noalloc(_ptr(z), DTYPES[dtype], G, m, n, C, _ptr(prev_masks),
+                                        _ptr(unit_group), U, _ptr(track), ctypes.byref(params),
+                                        _ptr(idx), _ptr(count), _ptr(status), _stream(stream))
+    _check(rc, "rs3_select_queries_noalloc")
 
 
 def rs3_memory_readout(q, dtype: str, G: int, mn: int, H: int, d: int, unit_group, idx, count,
