@@ -59,7 +59,8 @@ typedef enum {
     RS3_ECAPACITY = 2,     /* bank or workspace too small */
     RS3_EUNSUPPORTED = 3,  /* valid but not implemented (dtype / head dim / grid size) */
     RS3_ECUDA = 4,         /* a CUDA launch or query failed */
-    RS3_EINTERNAL = 5      /* inconsistent bank metadata */
+    RS3_EINTERNAL = 5,     /* inconsistent bank metadata */
+    RS3_ETIMEOUT = 6       /* a device-side wait gave up (status word only) */
 } rs3_status;
 
 typedef enum { RS3_F32 = 0, RS3_BF16 = 1 } rs3_dtype;
@@ -214,7 +215,8 @@ rs3_status rs3_bank_layout(int U, int H, int d, rs3_dtype dtype, int mn, int n_c
                            int64_t ring_cap_rows, int max_frames, int n_ptr,
                            int64_t *rows_per_unit, size_t *meta_bytes);
 
-/* Fills *bank and clears `meta` on `stream` (the banks start empty).
+/* Fills *bank and clears `meta`, `k_store` and `v_store` on `stream` (the
+ * banks start empty; storage rows never written read as zeros).
  * k_store / v_store: device [U][rows_per_unit][H*d]; meta: device, meta_bytes. */
 rs3_status rs3_bank_init(rs3_bank *bank, int U, int H, int d, rs3_dtype dtype, int mn, int n_cond,
                          int window, int64_t ring_cap_rows, int max_frames, int n_ptr,

@@ -33,6 +33,7 @@ extern "C" const char *rs3_status_string(int code)
     case RS3_EUNSUPPORTED: return "unsupported size or dtype";
     case RS3_ECUDA: return "CUDA error";
     case RS3_EINTERNAL: return "inconsistent bank metadata";
+    case RS3_ETIMEOUT: return "device wait timed out";
     default: return "unknown status";
     }
 }

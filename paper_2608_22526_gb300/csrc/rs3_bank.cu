@@ -251,7 +251,11 @@ extern "C" rs3_status rs3_bank_init(rs3_bank *bank, int U, int H, int d, rs3_dty
     bank->meta_stride = bank_meta_words(max_frames) * 8;
     bank->k_store = k_store; bank->v_store = v_store; bank->meta = meta;
     bank->magic = RS3_BANK_MAGIC;
-    if (cudaMemsetAsync(meta, 0, mb, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const size_t store_bytes = (size_t)U * (size_t)rows * (size_t)H * d * elem_bytes(dtype);
+    if (cudaMemsetAsync(meta, 0, mb, st) != cudaSuccess ||
+        cudaMemsetAsync(k_store, 0, store_bytes, st) != cudaSuccess ||
+        cudaMemsetAsync(v_store, 0, store_bytes, st) != cudaSuccess)
         return RS3_ECUDA;
     return RS3_OK;
 }

@@ -137,6 +137,11 @@ __global__ void __launch_bounds__(1024) k_plan(ReadoutArgs a)
             latch_status(a.status, RS3_EINVAL);
             cnt = cnt < 0 ? 0 : a.k_max;
         }
+        const int g = a.unit_group[u];
+        if (g < 0 || g >= a.G) {                    // no work for a unit without a valid grid
+            latch_status(a.status, RS3_EINVAL);
+            cnt = 0;
+        }
         const int64_t *mu = a.meta + (int64_t)u * a.meta_stride_words;
         const bool sane = mu[BM_HEAD] >= 0 && mu[BM_TAIL] >= mu[BM_HEAD] &&
                           mu[BM_TAIL] - mu[BM_HEAD] <= a.ring_cap && mu[BM_COND_LEN] >= 0 &&
@@ -500,6 +505,7 @@ rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, in
     a->n_sm = rs3_sm_count();
     a->min_chunk = p.kind == 1 ? 2 : 4;
     a->max_slots = L.max_slots;
+    a->max_items = L.max_items;
     const float sc = scale > 0.f ? scale : 1.0f / sqrtf((float)d);
     a->scale_log2 = sc * 1.4426950408889634f;
     a->header = reinterpret_cast<ReadoutHeader *>(ws + L.header);

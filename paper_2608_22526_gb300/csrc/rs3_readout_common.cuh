@@ -24,6 +24,7 @@ struct ReadoutArgs {
     int U, G, mn, H, d, D, k_max;
     int BM, BN, n_sm, min_chunk;
     int64_t max_slots;
+    int64_t max_items;
     float scale_log2;       // softmax scale * log2(e)
     ReadoutHeader *header;
     RangeSet *ranges;

@@ -15,7 +15,7 @@ import torch
 PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(PKG, "librs3.so")
 
-RS3_OK, RS3_EINVAL, RS3_ECAPACITY, RS3_EUNSUPPORTED, RS3_ECUDA, RS3_EINTERNAL = range(6)
+RS3_OK, RS3_EINVAL, RS3_ECAPACITY, RS3_EUNSUPPORTED, RS3_ECUDA, RS3_EINTERNAL, RS3_ETIMEOUT = range(7)
 RS3_F32, RS3_BF16 = 0, 1
 DTYPES = {"f32": RS3_F32, "bf16": RS3_BF16}
 TORCH_DTYPES = {"f32": torch.float32, "bf16": torch.bfloat16}
