@@ -429,7 +429,7 @@ def _traffic_record(w):
 def readout_source_hash():
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_22526_gb300", "csrc")
-    for f in ("rs3_readout.cu", "rs3_readout_tc.cu", "rs3_readout_common.cuh"):
+    for f in ("rs3_readout.cu", "rs3_readout_tc.cu", "rs3_readout_common.cuh", "rs3_tc_ptx.cuh"):
         p = os.path.join(csrc, f)
         if os.path.exists(p):
             h.update(open(p, "rb").read())

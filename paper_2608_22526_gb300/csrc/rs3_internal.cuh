@@ -75,7 +75,7 @@ struct ReadoutHeader {
 };
 
 struct ReadoutLayout {      // byte offsets inside the workspace
-    size_t header, ranges, items, combine, part_o, part_ml, total;
+    size_t header, cta_items, ranges, items, combine, part_o, part_ml, total;
     int64_t max_items, max_combine, max_slots;
 };
 

@@ -68,35 +68,6 @@ __device__ RangeSet unit_ranges(const ReadoutArgs &a, int u, int cnt)
     return rs;
 }
 
-__device__ __forceinline__ int splits_for(int n_tiles, int64_t chunk)
-{
-    if (n_tiles <= 1) return 1;
-    int64_t s = (n_tiles + chunk - 1) / chunk;
-    if (s > RS3_MAX_SPLITS) s = RS3_MAX_SPLITS;
-    if (s > n_tiles) s = n_tiles;
-    return s < 1 ? 1 : (int)s;
-}
-
-__device__ int64_t block_sum64(int64_t v)
-{
-    __shared__ int64_t s_part[32];
-    __shared__ int64_t s_tot;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    if (lane == 0) s_part[warp] = v;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        int64_t t = 0;
-        for (int w = 0; w < nw; ++w) t += s_part[w];
-        s_tot = t;
-    }
-    __syncthreads();
-    const int64_t r = s_tot;
-    __syncthreads();
-    return r;
-}
-
 // exclusive scan of an int64 per thread, returns offset; *total = block total
 __device__ int64_t block_scan64(int64_t v, int64_t *total)
 {
@@ -127,10 +98,90 @@ __device__ int64_t block_scan64(int64_t v, int64_t *total)
     return off;
 }
 
+// Stream-K plan.  Group g = (unit u, query tile qt, head h) owns
+// wg_u = max(T_u, 1) consecutive slots of a linear work axis (T_u = key tiles
+// of the unit's bank; an empty bank keeps one slot so its rows are written).
+// CTA b of P takes slots [b W / P, (b+1) W / P) and its slice is cut at group
+// boundaries into items.  A group that a slice boundary cuts is split: its
+// pieces write partials to consecutive slots (CTA order) and the CTA holding
+// its first piece emits the combine entry.
+struct PlanView {
+    const int64_t *tb;   // [U+1] first linear slot of each unit
+    const int64_t *wg;   // [U]   slots per group of each unit
+    int U, H;
+    int64_t W;
+    int P;
+};
+
+__device__ __forceinline__ int64_t slice_begin(const PlanView &v, int b)
+{
+    return (int64_t)b * v.W / v.P;
+}
+
+__device__ __forceinline__ void locate(const PlanView &v, int64_t x, int &u, int &gl, int64_t &off)
+{
+    int lo = 0, hi = v.U;                          // largest u with tb[u] <= x
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (v.tb[mid] <= x) lo = mid; else hi = mid;
+    }
+    u = lo;
+    const int64_t rel = x - v.tb[u];
+    gl = (int)(rel / v.wg[u]);
+    off = rel - (int64_t)gl * v.wg[u];
+}
+
+// Walks CTA b's slice; with write == false only counts items, partial items
+// and combine entries.
+__device__ void plan_slice(const ReadoutArgs &a, const PlanView &v, int b, bool write, int64_t item0,
+                           int64_t slot0, int64_t comb0, int &n_items, int &n_part, int &n_comb)
+{
+    n_items = n_part = n_comb = 0;
+    const int64_t lo = slice_begin(v, b), hi = slice_begin(v, b + 1);
+    for (int64_t x = lo; x < hi;) {
+        int u, gl;
+        int64_t off;
+        locate(v, x, u, gl, off);
+        const int64_t wg = v.wg[u];
+        const int64_t len = min(hi - x, wg - off);
+        const bool whole = off == 0 && len == wg;
+        if (write) {
+            const RangeSet &rs = a.ranges[u];
+            WorkItem w;
+            w.u = u; w.qt = gl / v.H; w.h = gl % v.H; w.split = 0;
+            w.tile_begin = (int32_t)min(off, (int64_t)rs.n_tiles);
+            w.tile_end = (int32_t)min(off + len, (int64_t)rs.n_tiles);
+            w.slot = whole ? -1 : (int32_t)(slot0 + n_part);
+            w.pad = 0;
+            a.items[item0 + n_items] = w;
+            if (!whole && off == 0) {
+                // first piece of a split group: count the slices it spans
+                const int64_t gend = x + wg - 1;            // last slot of the group
+                int e = b;
+                while (e + 1 < v.P && slice_begin(v, e + 1) <= gend) ++e;
+                CombineItem c;
+                c.u = u; c.h = w.h; c.qt = w.qt;
+                c.slot0 = (int32_t)(slot0 + n_part);
+                c.nsplit = e - b + 1;
+                c.pad[0] = c.pad[1] = c.pad[2] = 0;
+                a.combine[comb0 + n_comb] = c;
+            }
+        }
+        ++n_items;
+        if (!whole) {
+            if (off == 0) ++n_comb;
+            ++n_part;
+        }
+        x += len;
+    }
+}
+
 __global__ void __launch_bounds__(1024) k_plan(ReadoutArgs a)
 {
     ReadoutHeader *hdr = a.header;
-    int64_t work_local = 0;
+    extern __shared__ int64_t s_plan[];            // [U+1] tb, [U] wg, [3][grid+1] per-CTA counts
+    int64_t *s_tb = s_plan, *s_wg = s_plan + (a.U + 1);
+    int64_t *s_ci = s_wg + a.U, *s_cp = s_ci + (a.grid_ctas + 1), *s_cc = s_cp + (a.grid_ctas + 1);
     for (int u = threadIdx.x; u < a.U; u += blockDim.x) {
         int cnt = a.count[u];
         if (cnt < 0 || cnt > a.k_max) {
@@ -156,71 +207,55 @@ __global__ void __launch_bounds__(1024) k_plan(ReadoutArgs a)
             rs = unit_ranges(a, u, cnt);
         }
         a.ranges[u] = rs;
-        work_local += (int64_t)rs.nq * a.H * (rs.n_tiles > 0 ? rs.n_tiles : 1);
+        s_wg[u] = rs.n_tiles > 0 ? rs.n_tiles : 1;
     }
-    const int64_t W = block_sum64(work_local);     // syncs: ranges visible
-    int64_t chunk = (W + a.n_sm - 1) / a.n_sm;
-    if (chunk < a.min_chunk) chunk = a.min_chunk;
-    for (int iter = 0; iter < 40; ++iter) {
-        int64_t slots_local = 0;
-        for (int u = threadIdx.x; u < a.U; u += blockDim.x) {
-            const RangeSet &rs = a.ranges[u];
-            const int s = splits_for(rs.n_tiles, chunk);
-            if (s > 1) slots_local += (int64_t)rs.nq * a.H * s;
-        }
-        const int64_t S = block_sum64(slots_local);
-        if (S <= a.max_slots) break;
-        chunk *= 2;
-    }
-    // offsets, rounds of blockDim units
-    int64_t item_run = 0, slot_run = 0, comb_run = 0;
+    __syncthreads();
+    // linear slot base of every unit (exclusive scan in rounds of blockDim)
+    int64_t run = 0;
     for (int u0 = 0; u0 < a.U; u0 += blockDim.x) {
         const int u = u0 + threadIdx.x;
-        int64_t ni = 0, ns = 0, nc = 0;
-        int s = 1;
-        if (u < a.U) {
-            s = splits_for(a.ranges[u].n_tiles, chunk);
-            ni = (int64_t)a.ranges[u].nq * a.H * s;
-            ns = s > 1 ? ni : 0;
-            nc = s > 1 ? (int64_t)a.ranges[u].nq * a.H : 0;
-        }
-        int64_t ti, ts, tc;
-        const int64_t oi = block_scan64(ni, &ti) + item_run;
-        const int64_t os = block_scan64(ns, &ts) + slot_run;
-        const int64_t oc = block_scan64(nc, &tc) + comb_run;
-        if (u < a.U) {
-            RangeSet rs = a.ranges[u];
-            rs.splits = s;
-            rs.slot_base = s > 1 ? (int32_t)os : -1;
-            a.ranges[u] = rs;
-            int64_t it = oi, ic = oc;
-            for (int qt = 0; qt < rs.nq; ++qt)
-                for (int h = 0; h < a.H; ++h) {
-                    const int32_t slot0 = s > 1 ? (int32_t)(os + ((int64_t)qt * a.H + h) * s) : -1;
-                    for (int sp = 0; sp < s; ++sp) {
-                        WorkItem w;
-                        w.u = u; w.h = h; w.qt = qt; w.split = sp;
-                        w.tile_begin = (int32_t)((int64_t)sp * rs.n_tiles / s);
-                        w.tile_end = (int32_t)((int64_t)(sp + 1) * rs.n_tiles / s);
-                        w.slot = s > 1 ? slot0 + sp : -1;
-                        w.pad = 0;
-                        a.items[it++] = w;
-                    }
-                    if (s > 1) {
-                        CombineItem c;
-                        c.u = u; c.h = h; c.qt = qt; c.slot0 = slot0; c.nsplit = s;
-                        c.pad[0] = c.pad[1] = c.pad[2] = 0;
-                        a.combine[ic++] = c;
-                    }
-                }
-        }
-        item_run += ti;
-        slot_run += ts;
-        comb_run += tc;
+        const int64_t w = u < a.U ? (int64_t)a.ranges[u].nq * a.H * s_wg[u] : 0;
+        int64_t tot;
+        const int64_t off = block_scan64(w, &tot) + run;
+        if (u < a.U) s_tb[u] = off;
+        run += tot;
     }
+    if (threadIdx.x == 0) s_tb[a.U] = run;
+    __syncthreads();
+    PlanView v;
+    v.tb = s_tb; v.wg = s_wg; v.U = a.U; v.H = a.H; v.W = run;
+    int64_t P = (run + a.min_chunk - 1) / a.min_chunk;
+    if (P > a.grid_ctas) P = a.grid_ctas;
+    v.P = (int)P;
+    // per-CTA counts, then exclusive scans into offsets
+    for (int b = threadIdx.x; b < v.P; b += blockDim.x) {
+        int ni, np, nc;
+        plan_slice(a, v, b, false, 0, 0, 0, ni, np, nc);
+        s_ci[b] = ni; s_cp[b] = np; s_cc[b] = nc;
+    }
+    __syncthreads();
+    int64_t ri = 0, rp = 0, rc = 0;
+    for (int b0 = 0; b0 < v.P; b0 += blockDim.x) {
+        const int b = b0 + threadIdx.x;
+        const int64_t ni = b < v.P ? s_ci[b] : 0, np = b < v.P ? s_cp[b] : 0, nc = b < v.P ? s_cc[b] : 0;
+        int64_t ti, tp, tc;
+        const int64_t oi = block_scan64(ni, &ti) + ri;
+        const int64_t op = block_scan64(np, &tp) + rp;
+        const int64_t oc = block_scan64(nc, &tc) + rc;
+        if (b < v.P) { s_ci[b] = oi; s_cp[b] = op; s_cc[b] = oc; }
+        ri += ti; rp += tp; rc += tc;
+    }
+    __syncthreads();
+    for (int b = threadIdx.x; b < v.P; b += blockDim.x) {
+        int ni, np, nc;
+        plan_slice(a, v, b, true, s_ci[b], s_cp[b], s_cc[b], ni, np, nc);
+    }
+    for (int b = threadIdx.x; b <= a.grid_ctas; b += blockDim.x)
+        a.cta_items[b] = (int32_t)(b < v.P ? s_ci[b] : ri);
     if (threadIdx.x == 0) {
-        hdr->n_items = (int32_t)item_run;
-        hdr->n_combine = (int32_t)comb_run;
+        hdr->n_items = (int32_t)ri;
+        hdr->n_combine = (int32_t)rc;
+        hdr->pad[0] = v.P;
     }
 }
 
@@ -241,8 +276,8 @@ __global__ void __launch_bounds__(512) k_readout_simt(ReadoutArgs a)
     const int TPR = d / 16;
     float *sK = sm;                      // [SIMT_BN][d]
     float *sV = sm + SIMT_BN * d;        // [SIMT_BN][d]
-    const int n_items = a.header->n_items;
-    for (int it = blockIdx.x; it < n_items; it += gridDim.x) {
+    const int it_end = a.cta_items[blockIdx.x + 1];
+    for (int it = a.cta_items[blockIdx.x]; it < it_end; ++it) {
         const WorkItem w = a.items[it];
         const RangeSet rs = a.ranges[w.u];
         const int r = threadIdx.x / TPR;
@@ -360,41 +395,49 @@ __global__ void __launch_bounds__(512) k_readout_simt(ReadoutArgs a)
 template <typename T>
 __global__ void __launch_bounds__(256) k_combine(ReadoutArgs a)
 {
-    const int n_comb = a.header->n_combine;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    // one warp per output row: lane s holds split s's (m, l); lanes then
+    // stride the columns, every split's partial loaded without waiting on the
+    // previous one
+    const int64_t n_rows = (int64_t)a.header->n_combine * a.BM;
+    const int lane = threadIdx.x & 31;
     const int d = a.d;
-    for (int ci = blockIdx.x; ci < n_comb; ci += gridDim.x) {
+    const float2 *pm = reinterpret_cast<const float2 *>(a.part_ml);
+    for (int64_t gr = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; gr < n_rows;
+         gr += ((int64_t)gridDim.x * blockDim.x) >> 5) {
+        const int ci = (int)(gr / a.BM), r = (int)(gr % a.BM);
         const CombineItem c = a.combine[ci];
-        const RangeSet rs = a.ranges[c.u];
-        const int rows = min(a.BM, rs.cnt - c.qt * a.BM);
-        for (int r = warp; r < rows; r += nw) {
-            const int j = c.qt * a.BM + r;
-            int cell = a.idx[(int64_t)c.u * a.k_max + j];
-            if (cell < 0 || cell >= a.mn) cell = 0;
-            const float2 *pm = reinterpret_cast<const float2 *>(a.part_ml);
-            float M = -INFINITY;
-            for (int s = 0; s < c.nsplit; ++s) M = fmaxf(M, pm[(int64_t)(c.slot0 + s) * a.BM + r].x);
-            float L = 0.f;
+        const int j = c.qt * a.BM + r;
+        if (j >= a.ranges[c.u].cnt) continue;          // warp-uniform
+        int cell = a.idx[(int64_t)c.u * a.k_max + j];
+        if (cell < 0 || cell >= a.mn) cell = 0;
+        const float2 *ml = pm + (int64_t)c.slot0 * a.BM + r;      // split s at ml[s * BM]
+        float M = -INFINITY;
+        for (int s = lane; s < c.nsplit; s += 32) M = fmaxf(M, ml[(int64_t)s * a.BM].x);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+        float L = 0.f;
+        if (M != -INFINITY)
+            for (int s = lane; s < c.nsplit; s += 32) {
+                const float2 v = ml[(int64_t)s * a.BM];
+                L += exp2f(v.x - M) * v.y;
+            }
+        L = warp_sum(L);
+        const float inv = L > 0.f ? 1.f / L : 0.f;
+        const int64_t sstride = (int64_t)a.BM * d;
+        for (int c4 = lane * 4; c4 < d; c4 += 128) {              // no warp collectives below
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            const float *base = a.part_o + ((int64_t)c.slot0 * a.BM + r) * d + c4;
+#pragma unroll 4
             for (int s = 0; s < c.nsplit; ++s) {
-                const float2 ml = pm[(int64_t)(c.slot0 + s) * a.BM + r];
-                L += (M == -INFINITY) ? 0.f : exp2f(ml.x - M) * ml.y;
+                const float ws = M == -INFINITY ? 0.f : exp2f(ml[(int64_t)s * a.BM].x - M);
+                const float4 po = __ldcs(reinterpret_cast<const float4 *>(base + s * sstride));
+                acc.x = fmaf(ws, po.x, acc.x);
+                acc.y = fmaf(ws, po.y, acc.y);
+                acc.z = fmaf(ws, po.z, acc.z);
+                acc.w = fmaf(ws, po.w, acc.w);
             }
-            const float inv = L > 0.f ? 1.f / L : 0.f;
-            for (int c4 = lane * 4; c4 < d; c4 += 128) {
-                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-                for (int s = 0; s < c.nsplit; ++s) {
-                    const float2 ml = pm[(int64_t)(c.slot0 + s) * a.BM + r];
-                    const float wgt = (M == -INFINITY) ? 0.f : exp2f(ml.x - M);
-                    const float4 po = *reinterpret_cast<const float4 *>(
-                        a.part_o + ((int64_t)(c.slot0 + s) * a.BM + r) * d + c4);
-                    acc.x = fmaf(wgt, po.x, acc.x);
-                    acc.y = fmaf(wgt, po.y, acc.y);
-                    acc.z = fmaf(wgt, po.z, acc.z);
-                    acc.w = fmaf(wgt, po.w, acc.w);
-                }
-                float o4[4] = {acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv};
-                store_out4<T>(a, c.u, cell, c.h * d + c4, o4);
-            }
+            float o4[4] = {acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv};
+            store_out4<T>(a, c.u, cell, c.h * d + c4, o4);
         }
     }
 }
@@ -406,16 +449,22 @@ __global__ void __launch_bounds__(256) k_combine(ReadoutArgs a)
 // ---------------------------------------------------------------------------
 namespace {
 
-ReadoutLayout readout_layout(int U, int H, int d, int k_max, int BM)
+// Bounds of the stream-K plan: items <= groups + CTAs (a slice boundary adds
+// at most one item); a CTA has at most two partial items; at most one combine
+// entry per CTA and per group.
+ReadoutLayout readout_layout(int U, int H, int d, int k_max, int BM, int grid)
 {
     ReadoutLayout L;
     const int64_t nq = k_max > 0 ? (k_max + BM - 1) / BM : 1;
-    L.max_slots = RS3_MAX_SLOTS;
-    L.max_combine = (int64_t)U * H * nq;
-    L.max_items = L.max_combine + L.max_slots;
+    const int64_t groups = (int64_t)U * H * nq;
+    L.max_slots = 2 * (int64_t)grid;
+    L.max_combine = groups < grid ? groups : grid;
+    L.max_items = groups + grid;
     size_t off = 0;
     L.header = off;
     off = align_up(off + sizeof(ReadoutHeader), 256);
+    L.cta_items = off;
+    off = align_up(off + (size_t)(grid + 1) * 4, 256);
     L.ranges = off;
     off = align_up(off + (size_t)U * sizeof(RangeSet), 256);
     L.items = off;
@@ -435,14 +484,17 @@ ReadoutLayout readout_layout(int U, int H, int d, int k_max, int BM)
 ReadoutPath choose_readout_path(rs3_dtype dtype, int d)
 {
     ReadoutPath p;
+    const int n_sm = rs3_sm_count();
     if (dtype == RS3_BF16 && rs3_tc_supported(d)) {
         p.kind = 1;
         p.BM = 128;
         p.BN = rs3_tc_block_n(d);
+        p.grid = n_sm;                 // one persistent CTA per SM
     } else {
         p.kind = 0;
         p.BM = SIMT_BM;
         p.BN = SIMT_BN;
+        p.grid = 4 * n_sm;
     }
     return p;
 }
@@ -451,7 +503,7 @@ extern "C" size_t rs3_readout_workspace_bytes(int U, int H, int d, int k_max, rs
 {
     if (U < 1 || H < 1 || d < 1 || k_max < 0) return 0;
     const ReadoutPath p = choose_readout_path(dtype, d);
-    return readout_layout(U, H, d, k_max, p.BM).total;
+    return readout_layout(U, H, d, k_max, p.BM, p.grid).total;
 }
 
 rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, int H, int d,
@@ -468,13 +520,13 @@ rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, in
     if (dtype != RS3_F32 && dtype != RS3_BF16) return RS3_EINVAL;
     if ((int)dtype != bank->dtype || H != bank->H || d != bank->d) return RS3_EINVAL;
     if (G < 1 || mn < 1 || H < 1 || d < 1 || k_max < 0) return RS3_EINVAL;
-    if (mn > RS3_MAX_MN) return RS3_EUNSUPPORTED;
+    if (mn > RS3_MAX_MN || bank->U > RS3_MAX_UNITS) return RS3_EUNSUPPORTED;
     if (d < 16 || d > 256 || (d & (d - 1)) != 0) return RS3_EUNSUPPORTED;
     if (!rs3_aligned16(q) || !rs3_aligned16(out) || !rs3_aligned16(workspace) ||
         (residual && !rs3_aligned16(residual)) || (rope && !rs3_aligned16(rope)))
         return RS3_EINVAL;
     const ReadoutPath p = choose_readout_path(dtype, d);
-    const ReadoutLayout L = readout_layout(bank->U, H, d, k_max, p.BM);
+    const ReadoutLayout L = readout_layout(bank->U, H, d, k_max, p.BM, p.grid);
     if (workspace_bytes < L.total) return RS3_ECAPACITY;
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     a->q = q;
@@ -506,6 +558,8 @@ rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, in
     a->min_chunk = p.kind == 1 ? 2 : 4;
     a->max_slots = L.max_slots;
     a->max_items = L.max_items;
+    a->grid_ctas = p.grid;
+    a->cta_items = reinterpret_cast<int32_t *>(ws + L.cta_items);
     const float sc = scale > 0.f ? scale : 1.0f / sqrtf((float)d);
     a->scale_log2 = sc * 1.4426950408889634f;
     a->header = reinterpret_cast<ReadoutHeader *>(ws + L.header);
@@ -532,17 +586,25 @@ rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_
                                                         static_cast<uint4 *>(a.out), nvec);
         if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     }
-    k_plan<<<1, 1024, 0, st>>>(a);
+    // plan shared memory: unit slot bases and widths, per-CTA counts
+    const size_t plan_smem = ((size_t)(2 * a.U + 1) + 3 * (size_t)(a.grid_ctas + 1)) * 8;
+    static size_t plan_attr = 0;
+    if (plan_smem > 48 * 1024 && plan_smem > plan_attr) {
+        if (cudaFuncSetAttribute(k_plan, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan_smem) !=
+            cudaSuccess)
+            return RS3_EUNSUPPORTED;
+        plan_attr = plan_smem;
+    }
+    k_plan<<<1, 1024, plan_smem, st>>>(a);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
+    (void)max_items;
     if (p.kind == 1) {
         const rs3_status s = rs3_launch_tc_readout(a, st);
         if (s != RS3_OK) return s;
     } else {
         const size_t smem = (size_t)2 * SIMT_BN * a.d * sizeof(float);
         const int threads = 2 * a.d;
-        int64_t blocks = max_items;
-        const int64_t cap = (int64_t)a.n_sm * 16;
-        if (blocks > cap) blocks = cap;
+        const int64_t blocks = a.grid_ctas;
         static bool attr_done = false;
         if (!attr_done) {
             const int most = 2 * SIMT_BN * 256 * (int)sizeof(float);
@@ -556,7 +618,7 @@ rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_
             k_readout_simt<float><<<(unsigned)blocks, threads, smem, st>>>(a);
         if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     }
-    int64_t cblocks = max_combine;
+    int64_t cblocks = (max_combine * a.BM + 7) / 8;     // one warp per partial row
     const int64_t ccap = (int64_t)a.n_sm * 8;
     if (cblocks > ccap) cblocks = ccap;
     if (cblocks < 1) cblocks = 1;

@@ -4,7 +4,7 @@
 
 #include "rs3_internal.cuh"
 
-#define RS3_MAX_SLOTS 512   // split-KV partial tiles the planner may use
+#define RS3_MAX_UNITS 4096  // units per readout call
 
 struct ReadoutArgs {
     const void *q;
@@ -25,6 +25,8 @@ struct ReadoutArgs {
     int BM, BN, n_sm, min_chunk;
     int64_t max_slots;
     int64_t max_items;
+    int grid_ctas;          // CTAs of the readout launch (the plan's slice count bound)
+    int32_t *cta_items;     // [grid_ctas + 1]: CTA b runs items [cta_items[b], cta_items[b+1])
     float scale_log2;       // softmax scale * log2(e)
     ReadoutHeader *header;
     RangeSet *ranges;
@@ -37,6 +39,7 @@ struct ReadoutArgs {
 struct ReadoutPath {
     int kind;   // 0 = CUDA-core, 1 = tensor-core (tcgen05)
     int BM, BN;
+    int grid;   // CTAs of the readout launch
 };
 
 ReadoutPath choose_readout_path(rs3_dtype dtype, int d);

@@ -4,224 +4,61 @@
 // the log2 domain.
 //
 // One persistent CTA per SM walks the planner's work items (unit, head,
-// 128-query tile, range of 128-key tiles).  Per CTA, 8 warps:
-//   warp 0      K producer: TMA of the key tile (d/64 boxes of 128 rows x 64)
+// 128-query tile, range of BN-key tiles).  Per CTA, 8 warps:
+//   warp 0      K producer: TMA of the key tile (d/64 boxes of BN rows x 64)
 //   warp 2      V producer: TMA of the value tile
 //   warp 1      TMEM allocation; one lane issues every MMA:
-//               S_j = Q K_j^T   (M 128, N 128, K d; A = Q, B = K, both K-major)
-//               O  += P_j V_j   (M 128, N d, K 128; A = P K-major, B = V MN-major)
-//               S is double-buffered in TMEM so S_{j+1} runs while the
-//               softmax of S_j is computed.
-//   warps 4-7   one thread per query row: gather the kept query rows (and
-//               rotate them by RoPE of their own cell, Eq. 7) into shared
-//               memory, softmax of S_j from TMEM, P_j to shared memory as bf16,
-//               O rescaled in TMEM only when the running max grows by more
-//               than 2^8, and the epilogue (O / l + residual, or split-KV
-//               partials).
-// TMEM: O in columns [0, d), S buffers at 256 and 384 (512 columns).
+//               S_j = Q K_j^T   (M 128, N BN, K d; A = Q, B = K, both K-major)
+//               O  += P_j V_j   (M 128, N d, K BN; A = P K-major, B = V MN-major)
+//               S and P are double-buffered, so S_{j+1} runs while the softmax
+//               of S_j is computed and P_{j+1} is written while PV_j runs.
+//   warps 4-7   one thread per query row: gather the kept query rows with
+//               cp.async into the swizzled Q tile (rotated by RoPE of their
+//               own cell, Eq. 7, when a table is given), softmax of S_j from
+//               TMEM, P_j to shared memory as bf16, O rescaled in TMEM only
+//               when the running max grows by more than 2^8, and the epilogue
+//               (O / l + residual, or split-KV partials).
+// Shapes: d = 256 uses 64-key tiles with 2 K/V stages, d = 128 uses 128-key
+// tiles with 2 stages, d = 64 uses 128-key tiles with 3 stages.
+// TMEM: O in columns [0, d), S buffers from column 256 (512 columns).
 // Every mbarrier wait is bounded (1 s of %globaltimer): on expiry the CTA
 // raises an abort flag, drains its copies and MMAs, frees TMEM and the launch
 // latches RS3_ETIMEOUT.
 #include "rs3_readout_common.cuh"
+#include "rs3_tc_ptx.cuh"
 
-#include <cuda.h>
 #include <cudaTypedefs.h>
 
 namespace tc {
 
 constexpr int BM = 128;
-constexpr int BN = 128;
 constexpr int NTHREADS = 256;
-constexpr uint64_t WAIT_LIMIT_NS = 1000000000ull;
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t S_COL0 = 256;
 
 template <int DH>
 struct Cfg {
-    static constexpr int KST = DH == 256 ? 1 : (DH == 128 ? 2 : 3);   // K / V stages
+    static constexpr int BN = DH == 256 ? 64 : 128;          // keys per tile
+    static constexpr int KST = DH == 64 ? 3 : 2;             // K / V stages
     static constexpr int QBYTES = BM * DH * 2;
-    static constexpr int KVBYTES = BN * DH * 2;                          // one stage
-    static constexpr int PBYTES = BM * BN * 2;
+    static constexpr int KVBYTES = BN * DH * 2;              // one stage
+    static constexpr int PBYTES = BM * BN * 2;               // one P buffer
     static constexpr int OFF_Q = 0;
     static constexpr int OFF_K = OFF_Q + QBYTES;
     static constexpr int OFF_V = OFF_K + KST * KVBYTES;
     static constexpr int OFF_P = OFF_V + KST * KVBYTES;
-    static constexpr int OFF_BAR = OFF_P + PBYTES;
-    static constexpr int NBAR = 4 * KST + 8;
+    static constexpr int OFF_BAR = OFF_P + 2 * PBYTES;
+    static constexpr int NBAR = 4 * KST + 10;
     static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
     static constexpr int SMEM = OFF_MISC + 16 + 1024;                  // + alignment slack
     // barrier indices
     static constexpr int B_KFULL = 0, B_KEMPTY = KST, B_VFULL = 2 * KST, B_VEMPTY = 3 * KST;
     static constexpr int B_SFULL = 4 * KST, B_SFREE = 4 * KST + 2, B_PFULL = 4 * KST + 4;
-    static constexpr int B_PVDONE = 4 * KST + 5, B_QFULL = 4 * KST + 6, B_DRAIN = 4 * KST + 7;
+    static constexpr int B_PVDONE = 4 * KST + 6, B_QFULL = 4 * KST + 8, B_DRAIN = 4 * KST + 9;
 };
-static_assert(Cfg<256>::SMEM <= 232448, "shared memory budget");
+static_assert(Cfg<256>::SMEM <= 232448 && Cfg<128>::SMEM <= 232448 && Cfg<64>::SMEM <= 232448,
+              "shared memory budget");
 
-// ---------------------------------------------------------------------------
-// PTX wrappers
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ uint32_t smem_u32(const void *p)
-{
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
-{
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar)
-{
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes)
-{
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity)
-{
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-__device__ __forceinline__ uint64_t gtimer()
-{
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-// Waits for the phase with parity `parity` to complete; gives up (and raises
-// the CTA's abort flag) after WAIT_LIMIT_NS, or at once if the flag is up.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag)
-{
-    if (mbar_try(bar, parity)) return true;
-    const uint64_t t0 = gtimer();
-    while (true) {
-        if (mbar_try(bar, parity)) return true;
-        if (*abort_flag) return false;
-        if (gtimer() - t0 > WAIT_LIMIT_NS) {
-            *abort_flag = 1;
-            return false;
-        }
-    }
-}
-
-// Bounded wait that ignores the abort flag (used to drain work in flight).
-__device__ __forceinline__ void mbar_drain(uint32_t bar, uint32_t parity)
-{
-    const uint64_t t0 = gtimer();
-    while (!mbar_try(bar, parity))
-        if (gtimer() - t0 > WAIT_LIMIT_NS) return;
-}
-
-__device__ __forceinline__ void fence_proxy_async()
-{
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
-        ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
-        : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-__device__ __forceinline__ void tc_commit(uint32_t bar)
-{
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-                 : "memory");
-}
-
-__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                       uint32_t accumulate)
-{
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
-        ::"r"(d_tmem), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t *r)
-{
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
-        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
-          "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
-          "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
-          "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr));
-}
-
-__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t *r)
-{
-    asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
-        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
-        "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};"
-        ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]),
-          "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
-          "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
-          "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
-          "r"(r[29]), "r"(r[30]), "r"(r[31])
-        : "memory");
-}
-
-__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
-
-// Shared-memory matrix descriptor, 128-byte swizzle (tcgen05 format: start
-// address, leading / stride byte offsets in 16-byte units, version 1 at bit 46,
-// swizzle mode 2 at bits 61-63).  K-major tiles: SBO = 1024 (8 rows of 128 B),
-// LBO unused.  MN-major tiles: LBO = distance between 64-element column
-// blocks, SBO = 1024 (8 rows).
-__device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo)
-{
-    uint64_t d = 0;
-    d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
-    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
-    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
-    d |= (uint64_t)1 << 46;
-    d |= (uint64_t)2 << 61;
-    return d;
-}
-
-// Instruction descriptor of kind::f16: bf16 A and B, fp32 D, A K-major,
-// B K-major or MN-major, N >> 3 at bit 17, M >> 4 at bit 24.
-__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool b_mn_major)
-{
-    return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
-           ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
-}
-
-// Byte offset of 16-byte chunk `ch` (of 8 bf16) in row `r` of a K-major tile
-// with `rows` rows stored as 128-byte-swizzled 64-column blocks.
-__device__ __forceinline__ uint32_t sw128_offset(int rows, int r, int ch)
-{
-    return (uint32_t)((ch >> 3) * rows * 128 + r * 128 + (((ch & 7) ^ (r & 7)) << 4));
-}
-
-// ---------------------------------------------------------------------------
-// the kernel
-// ---------------------------------------------------------------------------
 template <int DH>
 __global__ void __launch_bounds__(NTHREADS, 1)
 k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
@@ -229,6 +66,7 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
 {
     using C = Cfg<DH>;
     constexpr int KST = C::KST;
+    constexpr int BN = C::BN;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -247,12 +85,12 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             mbar_init(BAR(C::B_VFULL + s), 1);
             mbar_init(BAR(C::B_VEMPTY + s), 1);
         }
-        mbar_init(BAR(C::B_SFULL + 0), 1);
-        mbar_init(BAR(C::B_SFULL + 1), 1);
-        mbar_init(BAR(C::B_SFREE + 0), 128);
-        mbar_init(BAR(C::B_SFREE + 1), 128);
-        mbar_init(BAR(C::B_PFULL), 128);
-        mbar_init(BAR(C::B_PVDONE), 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(BAR(C::B_SFULL + b), 1);
+            mbar_init(BAR(C::B_SFREE + b), 128);
+            mbar_init(BAR(C::B_PFULL + b), 128);
+            mbar_init(BAR(C::B_PVDONE + b), 1);
+        }
         mbar_init(BAR(C::B_QFULL), 128);
         mbar_init(BAR(C::B_DRAIN), 1);
         *abort_flag = 0;
@@ -272,7 +110,8 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    const int n_items = a.header->n_items;
+    // this CTA's slice of the stream-K plan
+    const int it_begin = a.cta_items[blockIdx.x], it_end = a.cta_items[blockIdx.x + 1];
 
     if ((warp == 0 || warp == 2) && lane == 0) {
         // ------------------------------------------------------------------
@@ -284,7 +123,7 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
         const int b_full = is_k ? C::B_KFULL : C::B_VFULL;
         const int b_empty = is_k ? C::B_KEMPTY : C::B_VEMPTY;
         uint32_t cnt = 0;
-        for (int it = blockIdx.x; it < n_items && !*abort_flag; it += gridDim.x) {
+        for (int it = it_begin; it < it_end && !*abort_flag; ++it) {
             const WorkItem w = a.items[it];
             const RangeSet rs = a.ranges[w.u];
             for (int t = w.tile_begin; t < w.tile_end; ++t, ++cnt) {
@@ -320,9 +159,9 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             const uint32_t kb = sK + st * C::KVBYTES;
 #pragma unroll
             for (int kk = 0; kk < DH / 16; ++kk) {
-                const uint32_t off = (uint32_t)((kk >> 2) * (BM * 128) + (kk & 3) * 32);
+                const uint32_t offq = (uint32_t)((kk >> 2) * (BM * 128) + (kk & 3) * 32);
                 const uint32_t offk = (uint32_t)((kk >> 2) * (BN * 128) + (kk & 3) * 32);
-                tc_mma(tmem + S_COL0 + 128u * b, desc_sw128(sQ + off, 16, 1024),
+                tc_mma(tmem + S_COL0 + (uint32_t)BN * b, desc_sw128(sQ + offq, 16, 1024),
                        desc_sw128(kb + offk, 16, 1024), ID_S, kk > 0 ? 1u : 0u);
             }
             tc_commit(BAR(C::B_SFULL + b));
@@ -330,7 +169,7 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             return true;
         };
         bool ok = true;
-        for (int it = blockIdx.x; it < n_items && ok; it += gridDim.x) {
+        for (int it = it_begin; it < it_end && ok; ++it) {
             const WorkItem w = a.items[it];
             const int n = w.tile_end - w.tile_begin;
             if (n <= 0) continue;
@@ -339,21 +178,22 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             tc_fence_after();
             if (!issue_s(tcnt)) { ok = false; break; }
             for (int j = 0; j < n; ++j) {
-                const uint32_t tj = tcnt + (uint32_t)j;
+                const uint32_t tj = tcnt + (uint32_t)j, pb = tj & 1u;
                 if (j + 1 < n && !issue_s(tj + 1)) { ok = false; break; }
                 const uint32_t st = tj % KST;
-                if (!mbar_wait(BAR(C::B_PFULL), tj & 1u, abort_flag)) { ok = false; break; }
+                if (!mbar_wait(BAR(C::B_PFULL + pb), (tj >> 1) & 1u, abort_flag)) { ok = false; break; }
                 if (!mbar_wait(BAR(C::B_VFULL + st), (tj / KST) & 1u, abort_flag)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t vb = sV + st * C::KVBYTES;
+                const uint32_t pbase = sP + pb * C::PBYTES;
 #pragma unroll
                 for (int kk = 0; kk < BN / 16; ++kk) {
                     const uint32_t offp = (uint32_t)((kk >> 2) * (BM * 128) + (kk & 3) * 32);
-                    tc_mma(tmem, desc_sw128(sP + offp, 16, 1024),
+                    tc_mma(tmem, desc_sw128(pbase + offp, 16, 1024),
                            desc_sw128(vb + (uint32_t)kk * 2048u, BN * 128, 1024), ID_PV,
                            (j > 0 || kk > 0) ? 1u : 0u);
                 }
-                tc_commit(BAR(C::B_PVDONE));
+                tc_commit(BAR(C::B_PVDONE + pb));
                 tc_commit(BAR(C::B_VEMPTY + st));
             }
             tcnt += (uint32_t)n;
@@ -363,66 +203,68 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
         mbar_drain(BAR(C::B_DRAIN), 0);
     } else if (warp >= 4) {
         // ------------------------------------------------------------------
-        // softmax / correction / epilogue: thread = query row
+        // gather, softmax / correction, epilogue: thread = query row
         // ------------------------------------------------------------------
         const int r = threadIdx.x - 128;              // 0..127 = TMEM lane
         const int wq = warp - 4;                      // TMEM lane quarter
         const uint32_t tl = tmem + ((uint32_t)(32 * wq) << 16);
         constexpr int CPR = DH / 8;                   // 16-byte chunks per query row
-        constexpr int RPI = 32 / CPR;                 // rows per warp per step
-        constexpr int QIT = BM / (4 * RPI);           // steps per warp
+        constexpr int NCH = BM * CPR / 128;           // chunks gathered per thread
         uint32_t tcnt = 0;
         bool ok = true;
-        for (int it = blockIdx.x; it < n_items && ok; it += gridDim.x) {
+        for (int it = it_begin; it < it_end && ok; ++it) {
             const WorkItem w = a.items[it];
             const RangeSet rs = a.ranges[w.u];
             const int n = w.tile_end - w.tile_begin;
-            const int g = a.unit_group[w.u];
             if (n > 0) {
-                // gather q~ rows of this query tile into the swizzled Q tile
+                // gather the kept query rows of this tile: chunk e = r + 128 k
+                // is 16 bytes of row e / CPR; rows past count are zero-filled
+                const int g = a.unit_group[w.u];
                 const uint16_t *qg = static_cast<const uint16_t *>(a.q) + (int64_t)g * a.mn * a.D + w.h * DH;
-#pragma unroll 1
-                for (int i0 = 0; i0 < QIT; i0 += 8) {
-                    uint4 v[8];
-                    int rr[8];
+                int cellk[NCH];
 #pragma unroll
-                    for (int u8 = 0; u8 < 8; ++u8) {
-                        const int i = i0 + u8;
-                        v[u8] = make_uint4(0, 0, 0, 0);
-                        rr[u8] = -1;
-                        if (i < QIT) {
-                            const int row = (i * 4 + wq) * RPI + lane / CPR;
-                            const int ch = lane % CPR;
-                            rr[u8] = row;
-                            const int jrow = w.qt * BM + row;
-                            if (jrow < rs.cnt) {
-                                int cell = a.idx[(int64_t)w.u * a.k_max + jrow];
-                                cell = (cell < 0 || cell >= a.mn) ? 0 : cell;
-                                v[u8] = __ldg(reinterpret_cast<const uint4 *>(qg + (int64_t)cell * a.D + ch * 8));
-                                if (a.rope) {
-                                    const float4 *f = reinterpret_cast<const float4 *>(
-                                        a.rope + ((int64_t)cell * (DH / 2) + ch * 4) * 2);
-                                    const float4 f0 = __ldg(f), f1 = __ldg(f + 1);
-                                    const float cs[4] = {f0.x, f0.z, f1.x, f1.z};
-                                    const float sn[4] = {f0.y, f0.w, f1.y, f1.w};
-                                    uint32_t wv[4] = {v[u8].x, v[u8].y, v[u8].z, v[u8].w};
-#pragma unroll
-                                    for (int p = 0; p < 4; ++p) {
-                                        const float x0 = __uint_as_float(wv[p] << 16);
-                                        const float x1 = __uint_as_float(wv[p] & 0xffff0000u);
-                                        wv[p] = pack_bf16x2(x0 * cs[p] - x1 * sn[p], x0 * sn[p] + x1 * cs[p]);
-                                    }
-                                    v[u8] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
-                                }
-                            }
-                        }
+                for (int k = 0; k < NCH; ++k) {
+                    const int row = (r + 128 * k) / CPR;
+                    const int jrow = w.qt * BM + row;
+                    int cell = -1;
+                    if (jrow < rs.cnt) {
+                        cell = a.idx[(int64_t)w.u * a.k_max + jrow];
+                        cell = (cell < 0 || cell >= a.mn) ? 0 : cell;
                     }
+                    cellk[k] = cell;
+                }
 #pragma unroll
-                    for (int u8 = 0; u8 < 8; ++u8) {
-                        if (rr[u8] < 0) continue;
-                        const uint32_t off = sw128_offset(BM, rr[u8], lane % CPR);
-                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(sQ + off), "r"(v[u8].x),
-                                     "r"(v[u8].y), "r"(v[u8].z), "r"(v[u8].w) : "memory");
+                for (int k = 0; k < NCH; ++k) {
+                    const int e = r + 128 * k, row = e / CPR, ch = e % CPR;
+                    const int cell = cellk[k];
+                    const uint16_t *src = qg + (int64_t)(cell < 0 ? 0 : cell) * a.D + ch * 8;
+                    cp_async16(sQ + sw128_offset(BM, row, ch), src, cell < 0 ? 0u : 16u);
+                }
+                cp_async_wait_all();
+                if (a.rope) {
+                    // Eq. 7: rotate each pair by f[cell] of the query's own cell
+#pragma unroll 4
+                    for (int k = 0; k < NCH; ++k) {
+                        const int cell = cellk[k];
+                        if (cell < 0) continue;
+                        const int e = r + 128 * k, row = e / CPR, ch = e % CPR;
+                        const uint32_t sa = sQ + sw128_offset(BM, row, ch);
+                        uint32_t wv[4];
+                        asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                                     : "=r"(wv[0]), "=r"(wv[1]), "=r"(wv[2]), "=r"(wv[3]) : "r"(sa));
+                        const float4 *f = reinterpret_cast<const float4 *>(
+                            a.rope + ((int64_t)cell * (DH / 2) + ch * 4) * 2);
+                        const float4 f0 = __ldg(f), f1 = __ldg(f + 1);
+                        const float cs[4] = {f0.x, f0.z, f1.x, f1.z};
+                        const float sn[4] = {f0.y, f0.w, f1.y, f1.w};
+#pragma unroll
+                        for (int p = 0; p < 4; ++p) {
+                            const float x0 = __uint_as_float(wv[p] << 16);
+                            const float x1 = __uint_as_float(wv[p] & 0xffff0000u);
+                            wv[p] = pack_bf16x2(x0 * cs[p] - x1 * sn[p], x0 * sn[p] + x1 * cs[p]);
+                        }
+                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(sa), "r"(wv[0]),
+                                     "r"(wv[1]), "r"(wv[2]), "r"(wv[3]) : "memory");
                     }
                 }
                 fence_proxy_async();
@@ -445,37 +287,54 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
                 tile_rows(rs, w.tile_begin + j, BN, row0, nvalid);
                 uint32_t sr[BN];
 #pragma unroll
-                for (int c4 = 0; c4 < BN / 32; ++c4) tmem_ld32(tl + S_COL0 + 128u * b + 32u * c4, sr + 32 * c4);
+                for (int c4 = 0; c4 < BN / 32; ++c4) tmem_ld32(tl + S_COL0 + (uint32_t)BN * b + 32u * c4, sr + 32 * c4);
                 tmem_wait_ld();
                 tc_fence_before();
                 mbar_arrive(BAR(C::B_SFREE + b));
-                float s[BN];
+                // row max of the raw scores (the scale is positive, so it is
+                // applied once to the max); columns past the range end masked
+                const bool full = nvalid >= BN;
                 float mt = -INFINITY;
+                if (full) {
 #pragma unroll
-                for (int c = 0; c < BN; ++c) {
-                    s[c] = c < nvalid ? __uint_as_float(sr[c]) * a.scale_log2 : -INFINITY;
-                    mt = fmaxf(mt, s[c]);
+                    for (int c = 0; c < BN; ++c) mt = fmaxf(mt, __uint_as_float(sr[c]));
+                } else {
+#pragma unroll
+                    for (int c = 0; c < BN; ++c) mt = fmaxf(mt, c < nvalid ? __uint_as_float(sr[c]) : -INFINITY);
                 }
+                mt *= a.scale_log2;
                 const float m_new = (j == 0) ? mt : (mt > m_run + 8.0f ? mt : m_run);
+                const float neg_m = -m_new;
                 float rowsum = 0.f;
                 uint32_t pk[BN / 2];
 #pragma unroll
                 for (int c = 0; c < BN / 2; ++c) {
-                    const float p0 = exp2f(s[2 * c] - m_new);
-                    const float p1 = exp2f(s[2 * c + 1] - m_new);
+                    float p0 = ex2_approx(fmaf(__uint_as_float(sr[2 * c]), a.scale_log2, neg_m));
+                    float p1 = ex2_approx(fmaf(__uint_as_float(sr[2 * c + 1]), a.scale_log2, neg_m));
+                    if (!full) {
+                        p0 = 2 * c < nvalid ? p0 : 0.f;
+                        p1 = 2 * c + 1 < nvalid ? p1 : 0.f;
+                    }
                     rowsum += p0 + p1;
                     pk[c] = pack_bf16x2(p0, p1);
                 }
+                // P buffer b was last read by PV of tile tj - 2
+                if (!__all_sync(0xffffffffu, mbar_wait(BAR(C::B_PVDONE + b), ((tj >> 1) & 1u) ^ 1u, abort_flag))) {
+                    ok = false;
+                    break;
+                }
                 if (j > 0) {
-                    // P_{j-1} consumed and O final for tile j-1
-                    if (!__all_sync(0xffffffffu, mbar_wait(BAR(C::B_PVDONE), (tj - 1u) & 1u, abort_flag))) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
                     const bool grow = m_new != m_run;
                     const float alpha = grow ? exp2f(m_run - m_new) : 1.0f;
                     if (__any_sync(0xffffffffu, grow)) {
+                        // O must hold tile j-1 before it is rescaled
+                        const uint32_t tp = tj - 1u;
+                        if (!__all_sync(0xffffffffu,
+                                        mbar_wait(BAR(C::B_PVDONE + (tp & 1u)), (tp >> 1) & 1u, abort_flag))) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
 #pragma unroll 1
                         for (int c4 = 0; c4 < DH / 32; ++c4) {
                             uint32_t o[32];
@@ -491,20 +350,22 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
                 }
                 l_run += rowsum;
                 m_run = m_new;
+                const uint32_t pbase = sP + b * C::PBYTES;
 #pragma unroll
                 for (int cc = 0; cc < BN / 8; ++cc) {
                     const uint32_t off = sw128_offset(BM, r, cc);
-                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(sP + off), "r"(pk[4 * cc]),
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(pbase + off), "r"(pk[4 * cc]),
                                  "r"(pk[4 * cc + 1]), "r"(pk[4 * cc + 2]), "r"(pk[4 * cc + 3]) : "memory");
                 }
                 fence_proxy_async();
                 tc_fence_before();
-                mbar_arrive(BAR(C::B_PFULL));
+                mbar_arrive(BAR(C::B_PFULL + b));
             }
             if (!ok) break;
             if (n > 0) {
+                const uint32_t tlast = tcnt + (uint32_t)n - 1u;
                 if (!__all_sync(0xffffffffu,
-                                mbar_wait(BAR(C::B_PVDONE), (tcnt + (uint32_t)n - 1u) & 1u, abort_flag))) {
+                                mbar_wait(BAR(C::B_PVDONE + (tlast & 1u)), (tlast >> 1) & 1u, abort_flag))) {
                     ok = false;
                     break;
                 }
@@ -596,13 +457,13 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
     return fn;
 }
 
-bool make_kv_map(CUtensorMap *m, const void *store, int64_t D, int64_t rows)
+bool make_kv_map(CUtensorMap *m, const void *store, int64_t D, int64_t rows, int box_rows)
 {
     PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
     if (!enc) return false;
     const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
     const cuuint64_t strides[1] = {(cuuint64_t)D * 2};
-    const cuuint32_t box[2] = {64, (cuuint32_t)BN};
+    const cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
     const cuuint32_t es[2] = {1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(store), dims, strides, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -622,10 +483,10 @@ rs3_status launch(const ReadoutArgs &a, cudaStream_t st)
     const int64_t rows = (int64_t)a.U * a.rows_per_unit;
     if (rows >= (int64_t)1 << 31) return RS3_EUNSUPPORTED;
     CUtensorMap mk, mv;
-    if (!make_kv_map(&mk, a.k_store, a.D, rows) || !make_kv_map(&mv, a.v_store, a.D, rows)) return RS3_ECUDA;
-    int64_t grid = a.max_items;
-    if (grid > a.n_sm) grid = a.n_sm;
-    if (grid < 1) grid = 1;
+    if (!make_kv_map(&mk, a.k_store, a.D, rows, Cfg<DH>::BN) ||
+        !make_kv_map(&mv, a.v_store, a.D, rows, Cfg<DH>::BN))
+        return RS3_ECUDA;
+    const int64_t grid = a.grid_ctas;               // the plan's slices; unused ones exit at once
     k_readout_tc<DH><<<(unsigned)grid, NTHREADS, Cfg<DH>::SMEM, st>>>(a, mk, mv);
     return cudaGetLastError() == cudaSuccess ? RS3_OK : RS3_ECUDA;
 }
@@ -633,7 +494,15 @@ rs3_status launch(const ReadoutArgs &a, cudaStream_t st)
 }  // namespace tc
 
 bool rs3_tc_supported(int d) { return d == 64 || d == 128 || d == 256; }
-int rs3_tc_block_n(int d) { (void)d; return tc::BN; }
+
+int rs3_tc_block_n(int d)
+{
+    switch (d) {
+    case 64: return tc::Cfg<64>::BN;
+    case 128: return tc::Cfg<128>::BN;
+    default: return tc::Cfg<256>::BN;
+    }
+}
 
 rs3_status rs3_launch_tc_readout(const ReadoutArgs &a, cudaStream_t st)
 {

@@ -75,6 +75,14 @@ def test_long_video_split_kv_small():
     run_lockstep(w, check_frames={1, 40, 79}, rows_per_unit=64)
 
 
+def test_long_bank_single_query_tile_split_across_many_ctas():
+    """Few kept queries (one 128-row tile) over a long bank: the one group is
+    cut into more than 32 pieces whose partials the combine merges."""
+    import dataclasses
+    w = dataclasses.replace(synth.scaled(W["long_video"], frames=80), rho=0.03)
+    run_lockstep(w, check_frames={1, 79}, rows_per_unit=64)
+
+
 def test_dense_rho1_identity():
     """rho = 1, full prior, unpruned bank: every cell is selected in order and
     the readout is dense memory attention (Sec. 3.1, after Eq. 7)."""
