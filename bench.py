@@ -136,8 +136,13 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 
 class DeviceSequence:
-    """All inputs of one sequence, resident on the device (and pinned on the
-    host for the end-to-end leg)."""
+    """Inputs of one sequence, resident on the device (and pinned on the host
+    for the end-to-end leg).  Masks follow the whole trajectory; the token
+    grids and memory-encoder outputs of large workloads come from a pool of
+    `pool` frames cycled along the sequence (frame t uses slot t % pool), which
+    bounds host memory and generation time while the pool still exceeds L2."""
+
+    POOL_BYTES = 6 << 30
 
     def __init__(self, w, dense: bool, device):
         import torch
@@ -145,14 +150,17 @@ class DeviceSequence:
         seq = synth.Sequence(w)
         T = w.frames
         ug = w.unit_group()
+        esz = 2 if w.dtype == "bf16" else 4
+        per_frame = (w.G + 3 * w.U) * w.mn * w.D * esz
+        self.pool = max(1, min(T, self.POOL_BYTES // per_frame))
 
         def dev(x):
             if x.dtype == np.uint16:
                 return torch.from_numpy(x.view(np.int16)).view(torch.bfloat16)
             return torch.from_numpy(np.ascontiguousarray(x))
 
-        z = [seq.z(t) for t in range(T)]
-        kv = [seq.kv_new(t) for t in range(T)]
+        z = [seq.z(t) for t in range(self.pool)]
+        kv = [seq.kv_new(t) for t in range(self.pool)]
         masks = [seq.masks(t) for t in range(T)]
         self.host = {
             "z": dev(np.stack(z)).pin_memory(),
@@ -161,6 +169,7 @@ class DeviceSequence:
             "v": dev(np.stack([b for _, b in kv])).pin_memory(),
             "mask": torch.from_numpy(np.stack(masks)).pin_memory(),
         }
+        del z, kv
         if dense:
             self.host["prev"] = torch.ones_like(self.host["mask"]).pin_memory()
         else:
@@ -172,44 +181,100 @@ class DeviceSequence:
         self.masks_np = masks
         self.T = T
 
+    def frame(self, key, t):
+        """Device tensor of input `key` for frame t."""
+        if key in ("z", "x", "k", "v"):
+            return self.dev[key][t % self.pool]
+        return self.dev[key][t]
+
     def h2d(self, stream):
+        """Every frame's inputs of one sequence from pinned host memory."""
         import torch
         with torch.cuda.stream(stream):
-            for k in ("z", "x", "k", "v", "mask", "prev"):
+            for k in ("mask", "prev"):
                 self.dev[k].copy_(self.host[k], non_blocking=True)
+            for t in range(self.T):
+                s = t % self.pool
+                for k in ("z", "x", "k", "v"):
+                    self.dev[k][s].copy_(self.host[k][s], non_blocking=True)
 
     def bytes_in(self):
-        return sum(self.host[k].numel() * self.host[k].element_size()
-                   for k in ("z", "x", "k", "v", "mask", "prev"))
+        per = {k: self.host[k][0].numel() * self.host[k].element_size() for k in ("z", "x", "k", "v")}
+        return (self.T * sum(per.values()) +
+                sum(self.host[k].numel() * self.host[k].element_size() for k in ("mask", "prev")))
 
 
-def run_step(pipe, data, timers=None):
-    """One step: the whole sequence through the library (Algorithm 1's loop)."""
+OVERLAP = "readout"
+
+
+def run_step(pipe, data, timers=None, side=None):
+    """One step: the whole sequence through the library (Algorithm 1's loop).
+
+    The selection of frame t+1 needs only frame t+1's grid and frame t's mask,
+    so it is issued on `side`: with OVERLAP == "commit" it runs beside frame
+    t's commit (after frame t's readout, so the persistent readout always has
+    every SM), with "readout" beside the readout and commit, with "none" in
+    line on the main stream."""
     import torch
     w = pipe.w
     from paper_2608_22526_gb300 import rs3
+    main = torch.cuda.current_stream()
+    side = side if (side is not None and OVERLAP != "none") else main
     rs3.rs3_bank_reset(pipe.bank, -1)
     pipe.track.zero_()
-    D = data.dev
+    F = data.frame
+    fork = torch.cuda.Event()
+    fork.record(main)
+    side.wait_event(fork)
+    sel_ev, rd_ev, sel_t = {}, {}, {}
+
+    def issue_select(t, after=None):
+        # frame t's keep-set goes to buffer t % 2, last read by the readout of t - 2
+        if t - 2 in rd_ev:
+            side.wait_event(rd_ev[t - 2])
+        if after is not None:
+            side.wait_event(after)
+        pipe.use_buffer(t % 2)
+        if timers is not None:
+            sel_t[t] = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+            sel_t[t][0].record(side)
+        pipe.select(F("z", t), F("prev", t), stream=side)
+        ev = torch.cuda.Event(enable_timing=timers is not None)
+        ev.record(side)
+        sel_ev[t] = ev
+        if timers is not None:
+            sel_t[t][1] = ev
+
+    first = 1 if w.n_cond > 0 else 0
     for t in range(data.T):
         if t == 0 and w.n_cond > 0:
-            pipe.commit(D["k"][t], D["v"][t], D["mask"][t], 1)
+            pipe.commit(F("k", t), F("v", t), F("mask", t), 1)
             if data.ptr is not None:
                 pipe.set_pointers(*data.ptr)
             continue
+        if t == first:
+            issue_select(t)
+        if t + 1 < data.T and OVERLAP == "readout":
+            issue_select(t + 1)          # beside this frame's readout and commit
+        main.wait_event(sel_ev[t])
+        pipe.use_buffer(t % 2)
         if timers is not None:
-            e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
-            e[0].record()
-        pipe.select(D["z"][t], D["prev"][t])
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            e[0].record(main)
+        pipe.readout(F("z", t), F("x", t), F("x", t))
+        ev = torch.cuda.Event(enable_timing=timers is not None)
+        ev.record(main)
+        rd_ev[t] = ev
+        if t + 1 < data.T and OVERLAP != "readout":
+            issue_select(t + 1, after=ev)    # beside this frame's commit
+        pipe.commit(F("k", t), F("v", t), F("mask", t), 0)
         if timers is not None:
-            e[1].record()
-        pipe.readout(D["z"][t], D["x"][t], D["x"][t])
-        if timers is not None:
-            e[2].record()
-        pipe.commit(D["k"][t], D["v"][t], D["mask"][t], 0)
-        if timers is not None:
-            e[3].record()
-            timers.append((t, e))
+            e[1] = ev
+            e[2].record(main)
+            timers.append((t, [sel_t[t][0], sel_t[t][1], e[0], e[1], e[2]]))
+    join = torch.cuda.Event()
+    join.record(side)
+    main.wait_event(join)
 
 
 def frame_work(w, counts, bank_lens, kw_lens):
@@ -225,27 +290,27 @@ def work_model(pipe, data):
     import torch
     from paper_2608_22526_gb300 import rs3
     w = pipe.w
-    D = data.dev
+    F = data.frame
     rs3.rs3_bank_reset(pipe.bank, -1)
     pipe.track.zero_()
     out = []
     for t in range(data.T):
         if t == 0 and w.n_cond > 0:
-            pipe.commit(D["k"][t], D["v"][t], D["mask"][t], 1)
+            pipe.commit(F("k", t), F("v", t), F("mask", t), 1)
             if data.ptr is not None:
                 pipe.set_pointers(*data.ptr)
             continue
-        pipe.select(D["z"][t], D["prev"][t])
+        pipe.select(F("z", t), F("prev", t))
         meta, _ = rs3.rs3_bank_read_meta(pipe.bank)
         counts = pipe.count.cpu().tolist()
         lens = meta[:, 7].tolist()
-        x = D["x"][t].clone()
-        pipe.readout(D["z"][t], x, x)
+        x = F("x", t).clone()
+        pipe.readout(F("z", t), x, x)
         if pipe.dense:
             kwl = [w.mn] * w.U
         else:
             kwl = [int(v) for v in data.masks_np[t].astype(bool).sum(axis=1)]
-        pipe.commit(D["k"][t], D["v"][t], D["mask"][t], 0)
+        pipe.commit(F("k", t), F("v", t), F("mask", t), 0)
         out.append((t, counts, lens, kwl))
     torch.cuda.synchronize()
     return out
@@ -274,23 +339,24 @@ def gpu_arm(args):
     for mode in (["pruned", "dense"] if not args.no_dense else ["pruned"]):
         pipe, data = build(mode == "dense")
         stream = torch.cuda.Stream()
+        side = torch.cuda.Stream()      # selection of frame t+1 runs beside frame t
         with torch.cuda.stream(stream):
             # warm-up (also sets kernel attributes before capture)
             for _ in range(max(args.warmup, 1)):
-                run_step(pipe, data)
+                run_step(pipe, data, side=side)
             torch.cuda.synchronize()
             work = work_model(pipe, data)
             torch.cuda.synchronize()
-            # per-call timing pass (events on the launching stream)
+            # per-call timing pass (events on each call's launching stream)
             timers = []
-            run_step(pipe, data, timers)
+            run_step(pipe, data, timers, side=side)
             torch.cuda.synchronize()
             sel_ms = [t[1][0].elapsed_time(t[1][1]) for t in timers]
-            rd_ms = [t[1][1].elapsed_time(t[1][2]) for t in timers]
-            cm_ms = [t[1][2].elapsed_time(t[1][3]) for t in timers]
+            rd_ms = [t[1][2].elapsed_time(t[1][3]) for t in timers]
+            cm_ms = [t[1][3].elapsed_time(t[1][4]) for t in timers]
             graph = torch.cuda.CUDAGraph()
             with torch.cuda.graph(graph, stream=stream):
-                run_step(pipe, data)
+                run_step(pipe, data, side=side)
             for _ in range(args.warmup):
                 graph.replay()
             torch.cuda.synchronize()
@@ -312,7 +378,7 @@ def gpu_arm(args):
             assert int(pipe.status.item()) == 0, "device status word set"
             # end-to-end through the public API with host buffers
             e2e_s = None
-            if mode == "pruned" and not args.no_e2e:
+            if mode == "pruned" and not args.no_e2e and data.pool == data.T:
                 out_host = torch.empty_like(data.host["x"]).pin_memory()
                 for _ in range(2):
                     data.h2d(stream)
@@ -525,7 +591,10 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--overlap", default="readout", choices=["commit", "readout", "none"])
     args = ap.parse_args()
+    global OVERLAP
+    OVERLAP = args.overlap
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
     if args.impl == "reference":

@@ -1,13 +1,9 @@
 // rs3_bank.cu -- ragged per-unit memory bank and the write-pruned commit
 // (Sec. 3.2, Eq. 8; Algorithm 1's sparse write).
 //
-// A commit is two launches:
-//   k_commit_plan  one CTA per unit: counts the kept rows per 256-cell chunk,
-//                  decides eviction / capacity from the old counters, updates
-//                  the counters and the frame table, and leaves a copy plan.
-//   k_commit_copy  one CTA per (chunk, unit): ballot/popc ranks of the kept
-//                  cells inside the chunk, then warp-per-row 128-bit copies of
-//                  the K and V rows to their bank rows.
+// A commit is one launch (k_commit): a CTA per (128-cell chunk, unit) ranks
+// its kept cells with ballot/popc and copies their K and V rows with 128-bit
+// accesses; the last CTA of each unit publishes the new counters.
 #include "rs3_internal.cuh"
 
 #include <cstdlib>
@@ -37,78 +33,6 @@ BankDev bank_dev(const rs3_bank *b)
     return v;
 }
 
-__device__ __forceinline__ int32_t *chunk_prefix(int64_t *mu, int max_frames)
-{
-    return reinterpret_cast<int32_t *>(mu + BM_HEADER_WORDS + 2 * (int64_t)max_frames);
-}
-
-__global__ void __launch_bounds__(1024)
-k_commit_plan(const uint8_t *__restrict__ mask, int mn, int is_cond, BankDev bk, int32_t *status)
-{
-    __shared__ int32_t s_cnt[BM_CHUNK_WORDS * 2];
-    const int u = blockIdx.x;
-    int64_t *mu = bk.meta + (int64_t)u * bk.stride_words;
-    const int nchunks = (mn + COMMIT_CHUNK - 1) / COMMIT_CHUNK;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-    const uint8_t *Mu = mask ? mask + (size_t)u * mn : nullptr;
-    for (int ch = warp; ch < nchunks; ch += nw) {
-        int c = 0;
-        for (int i = ch * COMMIT_CHUNK + lane; i < min(mn, (ch + 1) * COMMIT_CHUNK); i += 32)
-            c += Mu ? (Mu[i] != 0) : 1;
-        c = warp_sum(c);
-        if (lane == 0) s_cnt[ch] = c;
-    }
-    __syncthreads();
-    if (threadIdx.x != 0) return;
-    int32_t *pref = chunk_prefix(mu, bk.max_frames);
-    int64_t L = 0;
-    for (int ch = 0; ch < nchunks; ++ch) {
-        pref[ch] = (int32_t)L;
-        L += s_cnt[ch];
-    }
-    int64_t *foff = mu + BM_HEADER_WORDS;
-    int64_t *flen = foff + bk.max_frames;
-    bool ok;
-    int64_t base = 0;
-    if (is_cond) {
-        ok = mu[BM_NCOND] < bk.n_cond && mu[BM_COND_LEN] + L <= bk.pinned_cap;
-        if (ok) {
-            base = mu[BM_COND_LEN];
-            mu[BM_COND_LEN] += L;
-            mu[BM_NCOND] += 1;
-        }
-    } else {
-        int64_t head = mu[BM_HEAD], tail = mu[BM_TAIL];
-        int64_t nf = mu[BM_NFRAMES], oldest = mu[BM_OLDEST];
-        if (head < 0 || tail < head || nf < 0 || nf > bk.max_frames || oldest < 0 ||
-            oldest >= bk.max_frames) {
-            latch_status(status, RS3_EINTERNAL);
-            mu[BM_PLAN_OK] = 0;
-            return;
-        }
-        if (bk.window > 0 && nf == bk.window) {      // evict the oldest ring frame
-            head += flen[oldest];
-            oldest = (oldest + 1) % bk.max_frames;
-            nf -= 1;
-        }
-        ok = nf < bk.max_frames && (tail - head) + L <= bk.ring_cap;
-        if (ok) {
-            const int64_t slot = (oldest + nf) % bk.max_frames;
-            foff[slot] = tail;
-            flen[slot] = L;
-            base = tail;
-            mu[BM_HEAD] = head;
-            mu[BM_TAIL] = tail + L;
-            mu[BM_NFRAMES] = nf + 1;
-            mu[BM_OLDEST] = oldest;
-        }
-    }
-    if (!ok) latch_status(status, RS3_ECAPACITY);
-    mu[BM_PLAN_OK] = ok ? 1 : 0;
-    mu[BM_PLAN_COND] = is_cond ? 1 : 0;
-    mu[BM_PLAN_BASE] = base;
-}
-
 // Copies `nvec` 16-byte words of one row (one warp).
 __device__ __forceinline__ void copy_row(uint4 *__restrict__ dk, uint4 *__restrict__ dv,
                                          const uint4 *__restrict__ sk, const uint4 *__restrict__ sv,
@@ -122,51 +46,153 @@ __device__ __forceinline__ void copy_row(uint4 *__restrict__ dk, uint4 *__restri
     }
 }
 
+// Number of nonzero bytes in a 16-byte word.
+__device__ __forceinline__ int nonzero_bytes(uint4 w)
+{
+    return (__popc(__vcmpne4(w.x, 0u)) + __popc(__vcmpne4(w.y, 0u)) + __popc(__vcmpne4(w.z, 0u)) +
+            __popc(__vcmpne4(w.w, 0u))) >> 3;
+}
+
+// The commit of one frame, in one launch: CTA (c, u) owns cells
+// [c * COMMIT_CHUNK, (c+1) * COMMIT_CHUNK) of unit u.  Every CTA reads the
+// unit's old counters, counts the unit's kept rows (and those before its
+// chunk), takes the same eviction / capacity decision, ranks its kept cells
+// with ballot/popc and copies their K and V rows with 128-bit loads and
+// stores, a warp per row.  The last CTA of the unit to finish (an arrival
+// count in the unit's metadata, after a fence) publishes the new counters and
+// the frame-table entry, so no CTA can see counters of the frame it copies.
 __global__ void __launch_bounds__(256)
-k_commit_copy(const uint8_t *__restrict__ k_new, const uint8_t *__restrict__ v_new,
-              const uint8_t *__restrict__ mask, int mn, int64_t row_bytes, BankDev bk,
-              uint8_t *__restrict__ k_store, uint8_t *__restrict__ v_store)
+k_commit(const uint8_t *__restrict__ k_new, const uint8_t *__restrict__ v_new,
+         const uint8_t *__restrict__ mask, int mn, int is_cond, int64_t row_bytes, BankDev bk,
+         uint8_t *__restrict__ k_store, uint8_t *__restrict__ v_store, int32_t *status)
 {
     __shared__ int32_t s_list[COMMIT_CHUNK];
-    __shared__ int32_t s_wtot[8];
+    __shared__ int32_t s_red[2][8];
+    __shared__ int s_last;
     const int u = blockIdx.y, ch = blockIdx.x;
-    const int64_t *mu = bk.meta + (int64_t)u * bk.stride_words;
-    if (mu[BM_PLAN_OK] == 0) return;
-    const bool cond = mu[BM_PLAN_COND] != 0;
-    const int64_t base = mu[BM_PLAN_BASE];
-    const int32_t pre = reinterpret_cast<const int32_t *>(mu + BM_HEADER_WORDS + 2 * (int64_t)bk.max_frames)[ch];
-
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int cell = ch * COMMIT_CHUNK + threadIdx.x;
-    const bool keep = cell < mn && (mask ? mask[(size_t)u * mn + cell] != 0 : true);
-    const uint32_t bal = __ballot_sync(0xffffffffu, keep);
-    if (lane == 0) s_wtot[warp] = __popc(bal);
+    int64_t *mu = bk.meta + (int64_t)u * bk.stride_words;
+    const uint8_t *Mu = mask ? mask + (size_t)u * mn : nullptr;
+    const int64_t head0 = mu[BM_HEAD], tail0 = mu[BM_TAIL];
+    const int64_t nf0 = mu[BM_NFRAMES], oldest0 = mu[BM_OLDEST];
+    const int64_t cond_len0 = mu[BM_COND_LEN], ncond0 = mu[BM_NCOND];
+    const int64_t *foff = mu + BM_HEADER_WORDS;
+    const int64_t *flen = foff + bk.max_frames;
+
+    // kept rows of the whole unit, and of the chunks before this one
+    int total = 0, before = 0;
+    if (Mu) {
+        // 16-byte loads when the unit's mask row is aligned, bytes for the rest
+        const int nvec16 = (reinterpret_cast<uintptr_t>(Mu) & 15u) == 0 ? (mn >> 4) : 0;
+        for (int i = threadIdx.x; i < nvec16; i += blockDim.x) {
+            const int c = nonzero_bytes(__ldg(reinterpret_cast<const uint4 *>(Mu) + i));
+            total += c;
+            if (i * 16 < ch * COMMIT_CHUNK) before += c;
+        }
+        for (int i = nvec16 * 16 + threadIdx.x; i < mn; i += blockDim.x) {
+            const int c = Mu[i] != 0;
+            total += c;
+            if (i < ch * COMMIT_CHUNK) before += c;
+        }
+    } else if (threadIdx.x == 0) {
+        total = mn;
+        before = ch * COMMIT_CHUNK;
+    }
+    total = warp_sum(total);
+    before = warp_sum(before);
+    if (lane == 0) { s_red[0][warp] = total; s_red[1][warp] = before; }
     __syncthreads();
-    int off = 0, nk = 0;
+    int64_t L = 0, pre = 0;
 #pragma unroll
-    for (int w = 0; w < 8; ++w) {
-        off += (w < warp) ? s_wtot[w] : 0;
-        nk += s_wtot[w];
+    for (int w = 0; w < 8; ++w) { L += s_red[0][w]; pre += s_red[1][w]; }
+
+    // the decision (identical in every CTA of the unit)
+    bool ok;
+    int64_t base = 0, head = head0, oldest = oldest0, nf = nf0;
+    if (is_cond) {
+        ok = ncond0 < bk.n_cond && cond_len0 + L <= bk.pinned_cap;
+        base = cond_len0;
+    } else {
+        const bool sane = head0 >= 0 && tail0 >= head0 && nf0 >= 0 && nf0 <= bk.max_frames &&
+                          oldest0 >= 0 && oldest0 < bk.max_frames;
+        if (!sane) {
+            if (threadIdx.x == 0 && ch == 0) latch_status(status, RS3_EINTERNAL);
+            ok = false;
+        } else {
+            if (bk.window > 0 && nf == bk.window) {      // evict the oldest ring frame
+                head += flen[oldest];
+                oldest = (oldest + 1) % bk.max_frames;
+                nf -= 1;
+            }
+            ok = nf < bk.max_frames && (tail0 - head) + L <= bk.ring_cap;
+            base = tail0;
+        }
     }
-    if (keep) {
-        uint32_t lm;
-        asm("mov.u32 %0, %%lanemask_lt;" : "=r"(lm));
-        s_list[off + __popc(bal & lm)] = cell;
+
+    if (ok) {
+        // ranks of the kept cells of this chunk (ballot / popc), then copies
+        const int cell = ch * COMMIT_CHUNK + threadIdx.x;
+        const bool keep = threadIdx.x < COMMIT_CHUNK && cell < mn && (Mu ? Mu[cell] != 0 : true);
+        const uint32_t bal = __ballot_sync(0xffffffffu, keep);
+        __syncthreads();
+        if (lane == 0) s_red[0][warp] = __popc(bal);
+        __syncthreads();
+        int off = 0, nk = 0;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+            off += (w < warp) ? s_red[0][w] : 0;
+            nk += s_red[0][w];
+        }
+        if (keep) {
+            uint32_t lm;
+            asm("mov.u32 %0, %%lanemask_lt;" : "=r"(lm));
+            s_list[off + __popc(bal & lm)] = cell;
+        }
+        __syncthreads();
+        const int nvec = (int)(row_bytes / 16);
+        const uint8_t *ksrc = k_new + (size_t)u * mn * row_bytes;
+        const uint8_t *vsrc = v_new + (size_t)u * mn * row_bytes;
+        uint8_t *kdst = k_store + (size_t)u * bk.rows_per_unit * row_bytes;
+        uint8_t *vdst = v_store + (size_t)u * bk.rows_per_unit * row_bytes;
+        for (int j = warp; j < nk; j += 8) {
+            const int64_t rank = pre + j;
+            const int64_t row = is_cond ? base + rank : bk.pinned_cap + (base + rank) % bk.ring_cap;
+            const int64_t c = s_list[j];
+            copy_row(reinterpret_cast<uint4 *>(kdst + row * row_bytes),
+                     reinterpret_cast<uint4 *>(vdst + row * row_bytes),
+                     reinterpret_cast<const uint4 *>(ksrc + c * row_bytes),
+                     reinterpret_cast<const uint4 *>(vsrc + c * row_bytes), nvec, lane);
+        }
+    }
+
+    // arrival; the last CTA of the unit publishes the new counters
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        unsigned long long *arrive = reinterpret_cast<unsigned long long *>(mu + BM_ARRIVE);
+        s_last = atomicAdd(arrive, 1ull) == (unsigned long long)(gridDim.x - 1);
     }
     __syncthreads();
-    const int nvec = (int)(row_bytes / 16);
-    const uint8_t *ksrc = k_new + (size_t)u * mn * row_bytes;
-    const uint8_t *vsrc = v_new + (size_t)u * mn * row_bytes;
-    uint8_t *kdst = k_store + (size_t)u * bk.rows_per_unit * row_bytes;
-    uint8_t *vdst = v_store + (size_t)u * bk.rows_per_unit * row_bytes;
-    for (int j = warp; j < nk; j += 8) {
-        const int64_t rank = (int64_t)pre + j;
-        const int64_t row = cond ? base + rank : bk.pinned_cap + (base + rank) % bk.ring_cap;
-        const int64_t c = s_list[j];
-        copy_row(reinterpret_cast<uint4 *>(kdst + row * row_bytes),
-                 reinterpret_cast<uint4 *>(vdst + row * row_bytes),
-                 reinterpret_cast<const uint4 *>(ksrc + c * row_bytes),
-                 reinterpret_cast<const uint4 *>(vsrc + c * row_bytes), nvec, lane);
+    if (!s_last || threadIdx.x != 0) return;
+    __threadfence();
+    mu[BM_ARRIVE] = 0;
+    if (!ok) {
+        if (is_cond || (head0 >= 0 && tail0 >= head0)) latch_status(status, RS3_ECAPACITY);
+        return;
+    }
+    if (is_cond) {
+        mu[BM_COND_LEN] = cond_len0 + L;
+        mu[BM_NCOND] = ncond0 + 1;
+    } else {
+        int64_t *fo = mu + BM_HEADER_WORDS;
+        int64_t *fl = fo + bk.max_frames;
+        const int64_t slot = (oldest + nf) % bk.max_frames;
+        fo[slot] = tail0;
+        fl[slot] = L;
+        mu[BM_HEAD] = head;
+        mu[BM_TAIL] = tail0 + L;
+        mu[BM_NFRAMES] = nf + 1;
+        mu[BM_OLDEST] = oldest;
     }
 }
 
@@ -271,13 +297,11 @@ extern "C" rs3_status rs3_bank_commit(const rs3_bank *bank, const void *k_new, c
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const BankDev bk = bank_dev(bank);
     const int mn = bank->mn;
-    k_commit_plan<<<bank->U, 1024, 0, st>>>(keep_mask, mn, is_cond, bk, status);
-    if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     const int nchunks = (mn + COMMIT_CHUNK - 1) / COMMIT_CHUNK;
     const int64_t row_bytes = (int64_t)bank->D * (int64_t)elem_bytes(bank->dtype);
-    k_commit_copy<<<dim3(nchunks, bank->U), 256, 0, st>>>(
-        static_cast<const uint8_t *>(k_new), static_cast<const uint8_t *>(v_new), keep_mask, mn,
-        row_bytes, bk, static_cast<uint8_t *>(bank->k_store), static_cast<uint8_t *>(bank->v_store));
+    k_commit<<<dim3(nchunks, bank->U), 256, 0, st>>>(
+        static_cast<const uint8_t *>(k_new), static_cast<const uint8_t *>(v_new), keep_mask, mn, is_cond,
+        row_bytes, bk, static_cast<uint8_t *>(bank->k_store), static_cast<uint8_t *>(bank->v_store), status);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     return RS3_OK;
 }

@@ -24,22 +24,17 @@ enum {
     BM_OLDEST = 4,      // frame-table slot of the oldest ring frame
     BM_NCOND = 5,       // pinned frames held
     BM_PTRLEN = 6,      // pointer rows held
-    // commit plan, written by the plan kernel for the copy kernel
-    BM_PLAN_OK = 8,     // 1 = copy this commit, 0 = dropped
-    BM_PLAN_COND = 9,   // 1 = destination is the pinned region
-    BM_PLAN_BASE = 10,  // destination: pinned row or ring logical position
-    BM_HEADER_WORDS = 16,
-    BM_CHUNK_WORDS = 64 // per-chunk row prefix of the commit (mn / 256 <= 64)
+    BM_ARRIVE = 8,      // CTAs of the running commit that have finished
+    BM_HEADER_WORDS = 16
 };
-// after the header: int64 foff[max_frames], int64 flen[max_frames],
-// then int32 chunk_prefix[BM_CHUNK_WORDS * 2] (as int64 words: BM_CHUNK_WORDS)
+// after the header: int64 foff[max_frames], int64 flen[max_frames]
 
 __host__ __device__ inline int64_t bank_meta_words(int max_frames)
 {
-    return (int64_t)BM_HEADER_WORDS + 2 * (int64_t)max_frames + BM_CHUNK_WORDS;
+    return (int64_t)BM_HEADER_WORDS + 2 * (int64_t)max_frames;
 }
 
-#define COMMIT_CHUNK 256
+#define COMMIT_CHUNK 128
 
 // ---------------------------------------------------------------------------
 // Readout work list (in the caller's workspace)
@@ -79,7 +74,6 @@ struct ReadoutLayout {      // byte offsets inside the workspace
     int64_t max_items, max_combine, max_slots;
 };
 
-#define RS3_MAX_SPLITS 16
 
 // ---------------------------------------------------------------------------
 // Device helpers

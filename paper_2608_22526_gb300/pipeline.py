@@ -27,8 +27,12 @@ class Pipeline:
         dev = self.device
         self.unit_group = torch.tensor(w.unit_group(), dtype=torch.int32, device=dev)
         self.track = torch.zeros((w.U, 6), dtype=torch.int32, device=dev)
-        self.idx = torch.zeros((w.U, max(self.k_max, 1)), dtype=torch.int32, device=dev)
-        self.count = torch.zeros(w.U, dtype=torch.int32, device=dev)
+        # two keep-set buffers, so the selection of frame t+1 can be issued
+        # while the readout of frame t still reads its own keep-set
+        self.idx_buf = [torch.zeros((w.U, max(self.k_max, 1)), dtype=torch.int32, device=dev)
+                        for _ in range(2)]
+        self.count_buf = [torch.zeros(w.U, dtype=torch.int32, device=dev) for _ in range(2)]
+        self.idx, self.count = self.idx_buf[0], self.count_buf[0]
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
         self.ws_select = torch.empty(rs3.rs3_select_workspace_bytes(w.G, w.U, w.m, w.n),
                                      dtype=torch.uint8, device=dev)
@@ -41,11 +45,15 @@ class Pipeline:
         self.stream = stream
 
     # -- library calls -------------------------------------------------------
-    def select(self, z: torch.Tensor, prev_masks: torch.Tensor):
+    def use_buffer(self, i: int):
+        """Selects which keep-set buffer the next select / readout use."""
+        self.idx, self.count = self.idx_buf[i], self.count_buf[i]
+
+    def select(self, z: torch.Tensor, prev_masks: torch.Tensor, stream=None):
         w = self.w
         rs3.rs3_select_queries(z, w.dtype, w.G, w.m, w.n, w.C, prev_masks, self.unit_group, w.U,
                                self.track, self.params, self.idx, self.count, self.ws_select,
-                               self.status, self.stream)
+                               self.status, stream if stream is not None else self.stream)
 
     def readout(self, q: torch.Tensor, residual: Optional[torch.Tensor], out: torch.Tensor,
                 rope: Optional[torch.Tensor] = None, scale: float = 0.0):
