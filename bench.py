@@ -30,7 +30,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "pruned readout frames/s & TFLOP/s vs dense (1 GB300); bank-commit HBM GB/s"
 WORKLOAD = "sam2_1obj"
-KERNELS_PER_READOUT_FRAME = 8     # prior, energy, select, plan, readout, combine, commit plan, commit copy
+KERNELS_PER_READOUT_FRAME = 7     # prior, energy, select, plan, readout, combine, commit
 
 
 def _peaks():
@@ -435,13 +435,7 @@ def gpu_arm(args):
         "vs_baseline": None,
         "dtype": w.dtype,
         "data": "synthetic (seeded SAM2-shaped drifting-ellipse sequence; no dataset)",
-        "config": {"workload": f"{w.name}: {w.m}x{w.n} grid, {w.H}x{w.d} heads, cond + {w.window} "
-                               f"recent write-pruned frames + {w.n_ptr} pointer rows, "
-                               f"{w.frames} frames per step, rho {w.rho}",
-                   "global_batch": world, "seq_len": w.frames,
-                   "parallelism": f"replicas x{world}",
-                   "l2": "inputs per step exceed L2 (no flush)",
-                   "timing": "CUDA graph of the whole sequence, CUDA events"},
+        "config": workload_config(w, world),
         "readout_tflops": round(step_flops * args.steps / (P["dev_s"]) / 1e12, 3),
         "roofline": {"bound": "tensor", "achieved": round(achieved_tflops, 3),
                      "peak": tc_burst, "unit": "TFLOP/s",
@@ -457,7 +451,7 @@ def gpu_arm(args):
         "mean_queries": round(float(np.mean([sum(c) for c in P["counts"]])), 1),
         "mean_bank_rows": round(float(np.mean([sum(n) for n in P["lens"]])), 1),
         "clocks": P["clocks"],
-        "gpu_launches": (1 + (3 if w.n_ptr > 0 else 2) + (w.frames - (1 if w.n_cond > 0 else 0))
+        "gpu_launches": (1 + (2 if w.n_ptr > 0 else 1) + (w.frames - (1 if w.n_cond > 0 else 0))
                          * KERNELS_PER_READOUT_FRAME) * args.steps,
     }
     if "dense" in results:
@@ -477,6 +471,18 @@ def gpu_arm(args):
     if world > 1:
         dist.barrier()
         dist.destroy_process_group()
+
+
+def workload_config(w, world):
+    """The `config` object of the JSON line (both arms)."""
+    bank = (f"cond + {w.window} recent write-pruned frames" if w.window > 0
+            else "unbounded write-pruned bank")
+    return {"workload": f"{w.name}: {w.U} unit(s) on {w.G} grid(s) of {w.m}x{w.n}, {w.H}x{w.d} heads, "
+                        f"{bank} + {w.n_ptr} pointer rows, {w.frames} frames per step, rho {w.rho}",
+            "global_batch": world, "seq_len": w.frames,
+            "parallelism": f"replicas x{world}",
+            "l2": "inputs per step exceed L2 (no flush)",
+            "timing": "CUDA graph of the whole sequence, CUDA events"}
 
 
 def _traffic_record(w):
@@ -569,8 +575,8 @@ def reference_arm(args):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(s / max(n, 1) * 1e3, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": w.name, "global_batch": 1, "seq_len": w.frames,
-                   "parallelism": "host cores"},
+        "config": dict(workload_config(w, world), parallelism="host cores (rank 0)",
+                       timing="host wall clock per frame"),
         "impl": "reference",
         "cpu_baseline": {"value": round(v, 4) if v else None, "unit": "frames/s",
                          "cores": threads, "kind": "oracle", "sample": desc},

@@ -72,6 +72,23 @@ __device__ __forceinline__ void tile_rows(const RangeSet &rs, int t, int BN, int
     }
 }
 
+// Same, reading the range set in place (global memory) instead of a local copy.
+__device__ __forceinline__ void tile_rows(const RangeSet *rs, int t, int BN, int64_t &row0, int &nvalid)
+{
+    row0 = 0;
+    nvalid = 0;
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+        const int tiles = __ldg(&rs->tiles[r]);
+        if (t < tiles) {
+            row0 = __ldg(&rs->start[r]) + (int64_t)t * BN;
+            nvalid = min(BN, __ldg(&rs->len[r]) - t * BN);
+            return;
+        }
+        t -= tiles;
+    }
+}
+
 __device__ __forceinline__ float4 load4(const float *p) { return __ldg(reinterpret_cast<const float4 *>(p)); }
 __device__ __forceinline__ float4 load4(const uint16_t *p)
 {

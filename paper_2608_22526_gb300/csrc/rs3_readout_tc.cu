@@ -8,23 +8,26 @@
 //   warp 0      K producer: TMA of the key tile (d/64 boxes of BN rows x 64)
 //   warp 2      V producer: TMA of the value tile
 //   warp 1      TMEM allocation; one lane issues every MMA:
-//               S_j = Q K_j^T   (M 128, N BN, K d; A = Q, B = K, both K-major)
-//               O  += P_j V_j   (M 128, N d, K BN; A = P K-major, B = V MN-major)
-//               S and P are double-buffered, so S_{j+1} runs while the softmax
-//               of S_j is computed and P_{j+1} is written while PV_j runs.
-//   warps 4..   NSM softmax warpgroups.  Warp w reads TMEM lanes 32 (w % 4)..,
-//               i.e. query row r = 32 (w % 4) + lane; its group g = (w - 4) / 4
-//               owns columns [g CPT, (g+1) CPT) of S (CPT = 32 or 64) and
-//               columns [g d / NSM, (g+1) d / NSM) of O.  The groups gather
-//               the kept query rows with cp.async into the swizzled Q tile
-//               (rotated by RoPE of their own cell, Eq. 7, when a table is
-//               given), exchange row maxima through shared memory, write P_j
-//               as bf16, rescale O in TMEM only when the running max grows by
-//               more than 2^8, and run the epilogue (O / l + residual, or
-//               split-KV partials).
-// Shapes: d = 256 uses 64-key tiles with 2 K/V stages and 2 softmax groups,
-// d = 128 128-key tiles, 2 stages, 2 groups, d = 64 128-key tiles, 3 stages,
-// 4 groups.  TMEM: O in columns [0, d), S buffers from column 256 (512 columns).
+//               S_j = Q K_j^T   (M 128, N BN, K d; A = Q in TMEM, B = K tile,
+//                                K-major)
+//               O  += P_j V_j   (M 128, N d, K BN; A = P_j in shared memory,
+//                                B = V tile, MN-major)
+//               S runs two tiles ahead: S_{j+2} is queued as soon as the
+//               softmax has read S_j (two TMEM buffers), before PV_j.
+//   warps 4..   2 x 4 softmax warps; warps w and w + 4 own the same TMEM lane
+//               quarter (rows 32 (w % 4) + lane) and split the columns.  Per
+//               item each thread loads its slice of the kept query row,
+//               rotates it by the RoPE table of its own cell (Eq. 7) and
+//               writes it to TMEM as bf16 pairs; per tile it reads its slice
+//               of S_j, takes the exps against a running reference that moves
+//               only when the row max grows by more than 2^8 (O is then
+//               rescaled in TMEM), and writes P_j to shared memory (two
+//               buffers).  The slices of a row exchange their maxima through
+//               shared memory at a named barrier that also ANDs their wait
+//               results.  Epilogue: O / l + residual, or split-KV partials.
+// TMEM (512 columns): O in [0, d), S_0 / S_1 from S_COL, Q at Q_COL.
+// Shapes: d = 256 uses 64-key tiles, d = 128 and d = 64 128-key tiles; K and
+// V rings fill what shared memory leaves after the two P buffers.
 // Every mbarrier wait is bounded (1 s of %globaltimer): on expiry the CTA
 // raises an abort flag, drains its copies and MMAs, frees TMEM and the launch
 // latches RS3_ETIMEOUT.
@@ -37,65 +40,61 @@ namespace tc {
 
 constexpr int BM = 128;
 constexpr uint32_t TMEM_COLS = 512;
-constexpr uint32_t S_COL0 = 256;
 
 template <int DH>
 struct Cfg {
     static constexpr int BN = DH == 256 ? 64 : 128;          // keys per tile
-    static constexpr int KST = DH == 64 ? 3 : 2;             // K / V stages
-    static constexpr int NSM = 1;                            // softmax warpgroups
-    static constexpr int CPT = BN / NSM;                     // S columns per softmax thread
-    static constexpr int OCT = DH / NSM;                     // O columns per softmax thread
-    static constexpr int NTHREADS = 128 + 128 * NSM;
-    static constexpr int SMT = 128 * NSM;                    // softmax threads
-    static constexpr int QBYTES = BM * DH * 2;
-    static constexpr int KVBYTES = BN * DH * 2;              // one stage
+    static constexpr int KVBYTES = BN * DH * 2;              // one K (or V) stage
     static constexpr int PBYTES = BM * BN * 2;               // one P buffer
-    static constexpr int OFF_Q = 0;
-    static constexpr int OFF_K = OFF_Q + QBYTES;
-    static constexpr int OFF_V = OFF_K + KST * KVBYTES;
-    static constexpr int OFF_P = OFF_V + KST * KVBYTES;
-    static constexpr int OFF_RED = OFF_P + 2 * PBYTES;       // [NSM][128] floats
-    static constexpr int OFF_BAR = OFF_RED + NSM * BM * 4;
-    static constexpr int NBAR = 4 * KST + 11;
+    static constexpr int NSPLIT = 2;                         // softmax warps per TMEM lane quarter
+    // K stages, V stages: what the 227 KB of shared memory leave after the two
+    // P buffers, the row exchange, the barriers and the alignment slack
+    static constexpr int NKV = (232448 - 1024 - 16 - 64 * 8 - 3 * NSPLIT * BM * 4 - 2 * PBYTES) / KVBYTES;
+    static constexpr int KSTK = (NKV + 1) / 2, KSTV = NKV / 2;
+    static constexpr int NTHREADS = 128 + 128 * NSPLIT;
+    static constexpr int SCOLS = BN / NSPLIT;                // S columns of one softmax warp
+    static constexpr int PCOLS = SCOLS / 2;                  // its P pairs
+    static constexpr int OCOLS = DH / NSPLIT;                // its O columns
+    static constexpr int QCOLS = DH / 2 / NSPLIT;            // its Q columns (bf16 pairs)
+    static constexpr uint32_t S_COL = 256;                   // S_0 at S_COL, S_1 at S_COL + BN
+    static constexpr uint32_t Q_COL = DH == 256 ? 384 : DH;  // d/2 columns of bf16 pairs
+    static constexpr int OFF_K = 0;
+    static constexpr int OFF_V = OFF_K + KSTK * KVBYTES;
+    static constexpr int OFF_P = OFF_V + KSTV * KVBYTES;
+    static constexpr int OFF_RED = OFF_P + 2 * PBYTES;       // float [3][NSPLIT][BM]
+    static constexpr int OFF_BAR = OFF_RED + 3 * NSPLIT * BM * 4;
+    static constexpr int NBAR = 2 * KSTK + 2 * KSTV + 10;
     static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
-    static constexpr int SMEM = OFF_MISC + 16 + 1024;                  // + alignment slack
+    static constexpr int SMEM = OFF_MISC + 16 + 1024;        // + alignment slack
     // barrier indices
-    static constexpr int B_KFULL = 0, B_KEMPTY = KST, B_VFULL = 2 * KST, B_VEMPTY = 3 * KST;
-    static constexpr int B_SFULL = 4 * KST, B_SFREE = 4 * KST + 2, B_PFULL = 4 * KST + 4;
-    static constexpr int B_PVDONE = 4 * KST + 6, B_QFULL = 4 * KST + 8, B_DRAIN = 4 * KST + 9;
-    static constexpr int B_GRP = 4 * KST + 10;               // softmax groups' exchange barrier
-    static_assert(CPT % 32 == 0 && OCT % 16 == 0, "softmax slice shapes");
+    static constexpr int B_KFULL = 0, B_KEMPTY = KSTK, B_VFULL = 2 * KSTK, B_VEMPTY = 2 * KSTK + KSTV;
+    static constexpr int B_SFULL = 2 * KSTK + 2 * KSTV, B_SFREE = B_SFULL + 2, B_PFULL = B_SFULL + 4;
+    static constexpr int B_PVDONE = B_SFULL + 6, B_QFULL = B_SFULL + 8, B_DRAIN = B_SFULL + 9;
+    static_assert(S_COL + 2 * BN <= TMEM_COLS && Q_COL + DH / 2 <= TMEM_COLS, "TMEM budget");
+    static_assert(Q_COL >= (uint32_t)DH && (Q_COL + DH / 2 <= S_COL || Q_COL >= S_COL + 2 * BN), "TMEM overlap");
+    static_assert(SCOLS % 8 == 0 && PCOLS % 8 == 0 && QCOLS % 8 == 0 && OCOLS % 16 == 0, "warp slices");
+    static_assert(KSTK >= 2 && KSTV >= 2 && NBAR <= 64, "K/V stages");
 };
 static_assert(Cfg<256>::SMEM <= 232448 && Cfg<128>::SMEM <= 232448 && Cfg<64>::SMEM <= 232448,
               "shared memory budget");
 
-// Softmax pieces of one thread's S slice (raw scores as fp32 bits).
+// Softmax pieces of one row's S tile (raw scores as fp32 bits).
 template <int N>
-__device__ __forceinline__ float slice_max(const uint32_t (&sr)[N])
+__device__ __forceinline__ float row_max(const uint32_t (&sr)[N], int nv, bool full)
 {
     float m0 = -INFINITY, m1 = -INFINITY;
 #pragma unroll
     for (int c = 0; c < N; c += 2) {
-        m0 = fmaxf(m0, __uint_as_float(sr[c]));
-        m1 = fmaxf(m1, __uint_as_float(sr[c + 1]));
+        m0 = fmaxf(m0, (full || c < nv) ? __uint_as_float(sr[c]) : -INFINITY);
+        m1 = fmaxf(m1, (full || c + 1 < nv) ? __uint_as_float(sr[c + 1]) : -INFINITY);
     }
     return fmaxf(m0, m1);
 }
 
-template <int N>
-__device__ __forceinline__ float slice_max_masked(const uint32_t (&sr)[N], int nv)
-{
-    float m = -INFINITY;
-#pragma unroll
-    for (int c = 0; c < N; ++c) m = fmaxf(m, c < nv ? __uint_as_float(sr[c]) : -INFINITY);
-    return m;
-}
-
 // p = 2^(s * sc - ref) packed as bf16 pairs; returns the sum of the p.
 template <int N>
-__device__ __forceinline__ float slice_exp(const uint32_t (&sr)[N], uint32_t (&pk)[N / 2], float sc, float ref,
-                                           int nv, bool full)
+__device__ __forceinline__ float row_exp(const uint32_t (&sr)[N], uint32_t (&pk)[N / 2], float sc, float ref,
+                                         int nv, bool full)
 {
     const float nref = -ref;
     float r0 = 0.f, r1 = 0.f;
@@ -114,10 +113,10 @@ __device__ __forceinline__ float slice_exp(const uint32_t (&sr)[N], uint32_t (&p
     return r0 + r1;
 }
 
-// slice_exp against `ref`, and the max of the valid raw scores in the same pass.
+// row_exp against `ref`, and the max of the valid raw scores in the same pass.
 template <int N>
-__device__ __forceinline__ float slice_exp_max(const uint32_t (&sr)[N], uint32_t (&pk)[N / 2], float sc,
-                                               float ref, int nv, bool full, float &mx)
+__device__ __forceinline__ float row_exp_max(const uint32_t (&sr)[N], uint32_t (&pk)[N / 2], float sc,
+                                             float ref, int nv, bool full, float &mx)
 {
     const float nref = -ref;
     float r0 = 0.f, r1 = 0.f, m0 = -INFINITY, m1 = -INFINITY;
@@ -143,19 +142,49 @@ __device__ __forceinline__ float slice_exp_max(const uint32_t (&sr)[N], uint32_t
     return r0 + r1;
 }
 
+// NW consecutive bf16 pairs of one thread's kept query row -> its TMEM lane,
+// columns [tq, tq + NW) (element 2i in the low half).  With a RoPE table,
+// pair i is rotated by the (cos, sin) at rope[2i], rope[2i + 1] of the row's
+// own cell (Eq. 7).  qrow == nullptr writes zeros (rows past the kept count).
+template <int NW>
+__device__ __forceinline__ void q_pairs_to_tmem(const uint16_t *qrow, const float *rope, uint32_t tq)
+{
+    uint32_t w[NW];
+    if (qrow) {
+#pragma unroll
+        for (int i = 0; i < NW / 4; ++i) {
+            const uint4 v = __ldg(reinterpret_cast<const uint4 *>(qrow) + i);
+            w[4 * i] = v.x; w[4 * i + 1] = v.y; w[4 * i + 2] = v.z; w[4 * i + 3] = v.w;
+        }
+        if (rope) {
+#pragma unroll
+            for (int p = 0; p < NW; p += 2) {
+                const float4 f = __ldg(reinterpret_cast<const float4 *>(rope) + p / 2);
+                const float x0 = __uint_as_float(w[p] << 16), x1 = __uint_as_float(w[p] & 0xffff0000u);
+                const float y0 = __uint_as_float(w[p + 1] << 16), y1 = __uint_as_float(w[p + 1] & 0xffff0000u);
+                w[p] = pack_bf16x2(x0 * f.x - x1 * f.y, x0 * f.y + x1 * f.x);
+                w[p + 1] = pack_bf16x2(y0 * f.z - y1 * f.w, y0 * f.w + y1 * f.z);
+            }
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < NW; ++i) w[i] = 0u;
+    }
+    tmem_st_cols<NW>(tq, w);
+}
+
 template <int DH>
 __global__ void __launch_bounds__(Cfg<DH>::NTHREADS, 1)
 k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
              const __grid_constant__ CUtensorMap tmv)
 {
     using C = Cfg<DH>;
-    constexpr int KST = C::KST, BN = C::BN, NSM = C::NSM, CPT = C::CPT, OCT = C::OCT;
+    constexpr int KSTK = C::KSTK, KSTV = C::KSTV, BN = C::BN;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
     uint8_t *gbase = smem_raw + (base - raw);
-    const uint32_t sQ = base + C::OFF_Q, sK = base + C::OFF_K, sV = base + C::OFF_V, sP = base + C::OFF_P;
-    float *red = reinterpret_cast<float *>(gbase + C::OFF_RED);
+    const uint32_t sK = base + C::OFF_K, sV = base + C::OFF_V, sP = base + C::OFF_P;
     const uint32_t bars = base + C::OFF_BAR;
     volatile int *abort_flag = reinterpret_cast<volatile int *>(gbase + C::OFF_MISC);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(gbase + C::OFF_MISC + 8);
@@ -163,21 +192,22 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
 #define BAR(i) (bars + 8u * (uint32_t)(i))
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < KST; ++s) {
+        for (int s = 0; s < KSTK; ++s) {
             mbar_init(BAR(C::B_KFULL + s), 1);
             mbar_init(BAR(C::B_KEMPTY + s), 1);
+        }
+        for (int s = 0; s < KSTV; ++s) {
             mbar_init(BAR(C::B_VFULL + s), 1);
             mbar_init(BAR(C::B_VEMPTY + s), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(BAR(C::B_SFULL + b), 1);
-            mbar_init(BAR(C::B_SFREE + b), 4 * NSM);      // one arrival per softmax warp
-            mbar_init(BAR(C::B_PFULL + b), 4 * NSM);
+            mbar_init(BAR(C::B_SFREE + b), 4 * C::NSPLIT); // one arrival per softmax warp
+            mbar_init(BAR(C::B_PFULL + b), 4 * C::NSPLIT);
             mbar_init(BAR(C::B_PVDONE + b), 1);
         }
-        mbar_init(BAR(C::B_QFULL), 4 * NSM);
+        mbar_init(BAR(C::B_QFULL), 4 * C::NSPLIT);
         mbar_init(BAR(C::B_DRAIN), 1);
-        mbar_init(BAR(C::B_GRP), 4 * NSM);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         fence_proxy_async();
@@ -207,12 +237,13 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
         const uint32_t dst0 = is_k ? sK : sV;
         const int b_full = is_k ? C::B_KFULL : C::B_VFULL;
         const int b_empty = is_k ? C::B_KEMPTY : C::B_VEMPTY;
+        const uint32_t nst = is_k ? (uint32_t)KSTK : (uint32_t)KSTV;
         uint32_t cnt = 0;
         for (int it = it_begin; it < it_end && !*abort_flag; ++it) {
             const WorkItem w = a.items[it];
-            const RangeSet rs = a.ranges[w.u];
+            const RangeSet *rs = a.ranges + w.u;
             for (int t = w.tile_begin; t < w.tile_end; ++t, ++cnt) {
-                const uint32_t st = cnt % KST, ph = (cnt / KST) & 1u;
+                const uint32_t st = cnt % nst, ph = (cnt / nst) & 1u;
                 if (!mbar_wait(BAR(b_empty + st), ph ^ 1u, abort_flag)) goto producer_done;
                 int64_t row0;
                 int nvalid;
@@ -227,8 +258,8 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
         }
     producer_done:
         // let every copy this thread issued land before the CTA can exit
-        for (uint32_t k = (cnt > (uint32_t)KST ? cnt - KST : 0); k < cnt; ++k)
-            mbar_drain(BAR(b_full + k % KST), (k / KST) & 1u);
+        for (uint32_t k = (cnt > nst ? cnt - nst : 0); k < cnt; ++k)
+            mbar_drain(BAR(b_full + k % nst), (k / nst) & 1u);
     } else if (warp == 1 && lane == 0) {
         // ------------------------------------------------------------------
         // MMA issuer
@@ -238,28 +269,22 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
         // descriptors built once; a k-step only adds its byte offset / 16 to the
         // start-address field (every address stays below 256 KB, so the 14-bit
         // field cannot carry)
-        const uint64_t dq = desc_sw128(sQ, 16, 1024);
-        uint64_t dk[KST], dv[KST], dp[2];
-#pragma unroll
-        for (int s = 0; s < KST; ++s) {
-            dk[s] = desc_sw128(sK + s * C::KVBYTES, 16, 1024);
-            dv[s] = desc_sw128(sV + s * C::KVBYTES, BN * 128, 1024);
-        }
-        dp[0] = desc_sw128(sP, 16, 1024);
-        dp[1] = desc_sw128(sP + C::PBYTES, 16, 1024);
+        const uint64_t dk0 = desc_sw128(sK, 16, 1024), dv0 = desc_sw128(sV, BN * 128, 1024);
+        const uint64_t dp0 = desc_sw128(sP, 16, 1024);
+        constexpr uint32_t STAGE16 = C::KVBYTES >> 4, PBUF16 = C::PBYTES >> 4;
         uint32_t tcnt = 0, icnt = 0;
-        auto issue_s = [&](uint32_t tj) -> bool {
-            const uint32_t st = tj % KST, b = tj & 1u;
-            if (!mbar_wait(BAR(C::B_KFULL + st), (tj / KST) & 1u, abort_flag)) return false;
-            if (!mbar_wait(BAR(C::B_SFREE + b), ((tj >> 1) & 1u) ^ 1u, abort_flag)) return false;
+        // S_t = Q K_t^T into TMEM buffer t & 1, once the softmax has read S_{t-2}
+        auto issue_s = [&](uint32_t t) -> bool {
+            const uint32_t st = t % KSTK, b = t & 1u;
+            if (!mbar_wait(BAR(C::B_SFREE + b), ((t >> 1) & 1u) ^ 1u, abort_flag)) return false;
+            if (!mbar_wait(BAR(C::B_KFULL + st), (t / KSTK) & 1u, abort_flag)) return false;
             tc_fence_after();
-            const uint64_t dks = dk[st];
-            const uint32_t dst = tmem + S_COL0 + (uint32_t)BN * b;
+            const uint64_t dks = dk0 + st * STAGE16;
+            const uint32_t dst = tmem + C::S_COL + (uint32_t)BN * b;
 #pragma unroll
             for (int kk = 0; kk < DH / 16; ++kk) {
-                const uint32_t offq = (uint32_t)((kk >> 2) * (BM * 128) + (kk & 3) * 32);
                 const uint32_t offk = (uint32_t)((kk >> 2) * (BN * 128) + (kk & 3) * 32);
-                tc_mma(dst, dq + (offq >> 4), dks + (offk >> 4), ID_S, kk > 0 ? 1u : 0u);
+                tc_mma_ts(dst, tmem + C::Q_COL + 8u * kk, dks + (offk >> 4), ID_S, kk > 0 ? 1u : 0u);
             }
             tc_commit(BAR(C::B_SFULL + b));
             tc_commit(BAR(C::B_KEMPTY + st));
@@ -273,15 +298,18 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             if (!mbar_wait(BAR(C::B_QFULL), icnt & 1u, abort_flag)) { ok = false; break; }
             ++icnt;
             tc_fence_after();
+            // S runs two tiles ahead of PV: S_{j+2} is queued before PV_j, so
+            // the softmax of tile j+1 never waits for PV_j
             if (!issue_s(tcnt)) { ok = false; break; }
+            if (n > 1 && !issue_s(tcnt + 1)) { ok = false; break; }
             for (int j = 0; j < n; ++j) {
                 const uint32_t tj = tcnt + (uint32_t)j, pb = tj & 1u;
-                if (j + 1 < n && !issue_s(tj + 1)) { ok = false; break; }
-                const uint32_t st = tj % KST;
+                if (j + 2 < n && !issue_s(tj + 2)) { ok = false; break; }
+                const uint32_t st = tj % KSTV;
                 if (!mbar_wait(BAR(C::B_PFULL + pb), (tj >> 1) & 1u, abort_flag)) { ok = false; break; }
-                if (!mbar_wait(BAR(C::B_VFULL + st), (tj / KST) & 1u, abort_flag)) { ok = false; break; }
+                if (!mbar_wait(BAR(C::B_VFULL + st), (tj / KSTV) & 1u, abort_flag)) { ok = false; break; }
                 tc_fence_after();
-                const uint64_t dvs = dv[st], dps = dp[pb];
+                const uint64_t dvs = dv0 + st * STAGE16, dps = dp0 + pb * PBUF16;
 #pragma unroll
                 for (int kk = 0; kk < BN / 16; ++kk) {
                     const uint32_t offp = (uint32_t)((kk >> 2) * (BM * 128) + (kk & 3) * 32);
@@ -298,215 +326,154 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
         mbar_drain(BAR(C::B_DRAIN), 0);
     } else if (warp >= 4) {
         // ------------------------------------------------------------------
-        // gather, softmax / correction, epilogue
+        // query rows, softmax / correction, epilogue.  NSPLIT warps share a
+        // TMEM lane quarter (the same 32 rows, thread = row r); warp slice h
+        // owns columns [h SCOLS, (h+1) SCOLS) of S, the matching P pairs,
+        // O columns [h OCOLS, (h+1) OCOLS) and Q pairs [h QCOLS, (h+1) QCOLS).
+        // The slices of a row agree on the softmax reference through a named
+        // barrier per tile that also ANDs their wait results, so a timeout
+        // makes all of them leave together.
         // ------------------------------------------------------------------
-        const int ts = threadIdx.x - 128;             // 0 .. SMT-1
-        const int g = ts >> 7;                        // softmax group: column slice
-        const int wq = warp & 3;                      // TMEM lane quarter
-        const int r = 32 * wq + lane;                 // query row of the tile
-        const uint32_t tl = tmem + ((uint32_t)(32 * wq) << 16);
-        constexpr int CPR = DH / 8;                   // 16-byte chunks per query row
-        constexpr int NCH = BM * CPR / C::SMT;        // chunks gathered per thread
+        constexpr int NSPLIT = C::NSPLIT, SCOLS = C::SCOLS, PCOLS = C::PCOLS, OCOLS = C::OCOLS,
+                      QCOLS = C::QCOLS;
+        const int q4 = warp & 3, h = (warp - 4) >> 2;
+        const int r = 32 * q4 + lane;                 // query row of the tile
+        const uint32_t tl = tmem + ((uint32_t)(32 * q4) << 16);
+        const uint32_t bar_id = 1u + (uint32_t)q4, bar_n = 32u * NSPLIT;
+        float *red = reinterpret_cast<float *>(gbase + C::OFF_RED);   // [3][NSPLIT][BM]
         uint32_t tcnt = 0;
         bool ok = true;
-        float *red_r = red + r;                       // red[g * 128 + r]
-        // barrier of all softmax warps (one arrival per warp), bounded like
-        // every other wait so that an abort cannot strand a group
-        uint32_t grp_phase = 0;
-        auto grp_sync = [&]() -> bool {
-            __syncwarp();
-            if (lane == 0) mbar_arrive(BAR(C::B_GRP));
-            const bool okw = __all_sync(0xffffffffu, mbar_wait(BAR(C::B_GRP), grp_phase & 1u, abort_flag));
-            ++grp_phase;
-            return okw;
-        };
         for (int it = it_begin; it < it_end && ok; ++it) {
             const WorkItem w = a.items[it];
-            const RangeSet rs = a.ranges[w.u];
+            const RangeSet *rs = a.ranges + w.u;
             const int n = w.tile_end - w.tile_begin;
+            const int jrow = w.qt * BM + r;
+            const bool valid = jrow < __ldg(&rs->cnt);
+            int cell = valid ? a.idx[(int64_t)w.u * a.k_max + jrow] : 0;
+            cell = (cell < 0 || cell >= a.mn) ? 0 : cell;
             if (n > 0) {
-                // gather the kept query rows of this tile: chunk e = ts + SMT k
-                // is 16 bytes of row e / CPR; rows past count are zero-filled
+                // Q of the previous item is no longer read: its last PV, which
+                // completes after every earlier MMA, was waited for
                 const int gq = a.unit_group[w.u];
-                const uint16_t *qg = static_cast<const uint16_t *>(a.q) + (int64_t)gq * a.mn * a.D + w.h * DH;
-                int cellk[NCH];
-#pragma unroll
-                for (int k = 0; k < NCH; ++k) {
-                    const int row = (ts + C::SMT * k) / CPR;
-                    const int jrow = w.qt * BM + row;
-                    int cell = -1;
-                    if (jrow < rs.cnt) {
-                        cell = a.idx[(int64_t)w.u * a.k_max + jrow];
-                        cell = (cell < 0 || cell >= a.mn) ? 0 : cell;
-                    }
-                    cellk[k] = cell;
-                }
-#pragma unroll
-                for (int k = 0; k < NCH; ++k) {
-                    const int e = ts + C::SMT * k, row = e / CPR, ch = e % CPR;
-                    const int cell = cellk[k];
-                    const uint16_t *src = qg + (int64_t)(cell < 0 ? 0 : cell) * a.D + ch * 8;
-                    cp_async16(sQ + sw128_offset(BM, row, ch), src, cell < 0 ? 0u : 16u);
-                }
-                cp_async_wait_all();
-                if (a.rope) {
-                    // Eq. 7: rotate each pair by f[cell] of the query's own cell
-#pragma unroll
-                    for (int k = 0; k < NCH; ++k) {
-                        const int cell = cellk[k];
-                        if (cell < 0) continue;
-                        const int e = ts + C::SMT * k, row = e / CPR, ch = e % CPR;
-                        const uint32_t sa = sQ + sw128_offset(BM, row, ch);
-                        uint32_t wv[4];
-                        asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
-                                     : "=r"(wv[0]), "=r"(wv[1]), "=r"(wv[2]), "=r"(wv[3]) : "r"(sa));
-                        const float4 *f = reinterpret_cast<const float4 *>(
-                            a.rope + ((int64_t)cell * (DH / 2) + ch * 4) * 2);
-                        const float4 f0 = __ldg(f), f1 = __ldg(f + 1);
-                        const float cs[4] = {f0.x, f0.z, f1.x, f1.z};
-                        const float sn[4] = {f0.y, f0.w, f1.y, f1.w};
-#pragma unroll
-                        for (int p = 0; p < 4; ++p) {
-                            const float x0 = __uint_as_float(wv[p] << 16);
-                            const float x1 = __uint_as_float(wv[p] & 0xffff0000u);
-                            wv[p] = pack_bf16x2(x0 * cs[p] - x1 * sn[p], x0 * sn[p] + x1 * cs[p]);
-                        }
-                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(sa), "r"(wv[0]),
-                                     "r"(wv[1]), "r"(wv[2]), "r"(wv[3]) : "memory");
-                    }
-                }
-                fence_proxy_async();
+                const uint16_t *qrow = valid ? static_cast<const uint16_t *>(a.q) +
+                                                   ((int64_t)gq * a.mn + cell) * a.D + w.h * DH + 2 * h * QCOLS
+                                             : nullptr;
+                const float *rope = a.rope ? a.rope + (int64_t)cell * DH + 2 * h * QCOLS : nullptr;
+                q_pairs_to_tmem<QCOLS>(qrow, rope, tl + C::Q_COL + (uint32_t)(h * QCOLS));
+                tmem_wait_st();
+                tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(BAR(C::B_QFULL));
             }
-            const int jrow = w.qt * BM + r;
-            const bool valid = jrow < rs.cnt;
-            int cell = valid ? a.idx[(int64_t)w.u * a.k_max + jrow] : 0;
-            cell = (cell < 0 || cell >= a.mn) ? 0 : cell;
             float m_run = -INFINITY, l_part = 0.f;
             for (int j = 0; j < n; ++j) {
                 const uint32_t tj = tcnt + (uint32_t)j, b = tj & 1u;
-                if (!__all_sync(0xffffffffu, mbar_wait(BAR(C::B_SFULL + b), (tj >> 1) & 1u, abort_flag))) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
+                const bool okw = __all_sync(0xffffffffu, mbar_wait(BAR(C::B_SFULL + b), (tj >> 1) & 1u, abort_flag));
                 int64_t row0;
-                int nvalid;
-                tile_rows(rs, w.tile_begin + j, BN, row0, nvalid);
-                uint32_t sr[CPT];
-#pragma unroll
-                for (int c4 = 0; c4 < CPT / 32; ++c4)
-                    tmem_ld32(tl + S_COL0 + (uint32_t)BN * b + (uint32_t)(g * CPT) + 32u * c4, sr + 32 * c4);
-                tmem_wait_ld();
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(BAR(C::B_SFREE + b));
-                // Valid columns of this slice.  After the first tile of an item
-                // the exps are taken against the running reference m_run with
-                // the tile max gathered in the same pass; only if the max grows
-                // past m_run + 8 (a factor 2^8) are they redone against the new
-                // max (and O rescaled below).  The first tile takes its max
-                // first.  The scale is positive, so it is applied to the max of
-                // the raw scores.
-                const int nv = nvalid - g * CPT;      // may be <= 0 for a late slice
-                const bool full = nv >= CPT;
+                int nvt;
+                tile_rows(rs, w.tile_begin + j, BN, row0, nvt);
+                const int nv = nvt - h * SCOLS;       // valid columns of this slice (may be <= 0)
+                const bool full = nv >= SCOLS;
+                const uint32_t scol = tl + C::S_COL + (uint32_t)BN * b;
                 const float sc = a.scale_log2;
-                uint32_t pk[CPT / 2];
-                float rowsum, m_new;
-                if (j == 0 || NSM > 1) {
-                    float mt = full ? slice_max<CPT>(sr) : slice_max_masked<CPT>(sr, nv);
-                    if (NSM > 1) {
-                        red_r[g * BM] = mt;
-                        if (!grp_sync()) { ok = false; break; }
-#pragma unroll
-                        for (int q = 0; q < NSM; ++q) mt = fmaxf(mt, red_r[q * BM]);
-                        if (!grp_sync()) { ok = false; break; }
-                    }
-                    mt *= sc;
-                    m_new = (j == 0) ? mt : (mt > m_run + 8.0f ? mt : m_run);
-                    rowsum = slice_exp<CPT>(sr, pk, sc, m_new, nv, full);
+                uint32_t sr[SCOLS], pk[PCOLS];
+                float mt, rowsum = 0.f;
+                if (okw) {
+                    tc_fence_after();
+                    tmem_ld_cols<SCOLS>(scol + (uint32_t)(h * SCOLS), sr);
+                    tmem_wait_ld();
+                    // S_j is in registers: its TMEM buffer may take S_{j+2}
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(BAR(C::B_SFREE + b));
+                    // After the first tile of an item the exps are taken against
+                    // the running reference m_run, with the slice max gathered in
+                    // the same pass.  The scale is positive, so it is applied to
+                    // the max of the raw scores.
+                    if (j == 0) mt = row_max<SCOLS>(sr, nv, full);
+                    else rowsum = row_exp_max<SCOLS>(sr, pk, sc, m_run, nv, full, mt);
                 } else {
-                    float mt;
-                    rowsum = slice_exp_max<CPT>(sr, pk, sc, m_run, nv, full, mt);
-                    m_new = m_run;
-                    if (mt * sc > m_run + 8.0f) {
-                        m_new = mt * sc;
-                        rowsum = slice_exp<CPT>(sr, pk, sc, m_new, nv, full);
-                    }
+                    mt = -INFINITY;
                 }
-                // P buffer b was last read by PV of tile tj - 2
-                if (!__all_sync(0xffffffffu, mbar_wait(BAR(C::B_PVDONE + b), ((tj >> 1) & 1u) ^ 1u, abort_flag))) {
-                    ok = false;
-                    break;
+                float *redt = red + (b * NSPLIT) * BM;
+                redt[h * BM + r] = mt;
+                if (!bar_and(bar_id, bar_n, okw)) { ok = false; break; }
+                float mrow = redt[r];
+#pragma unroll
+                for (int q = 1; q < NSPLIT; ++q) mrow = fmaxf(mrow, redt[q * BM + r]);
+                // the first tile sets the reference; a later one moves it only if
+                // the row max grows past it by more than 2^8 (O is then rescaled)
+                float m_new = m_run;
+                if (j == 0 || mrow * sc > m_run + 8.0f) {
+                    m_new = mrow * sc;
+                    rowsum = row_exp<SCOLS>(sr, pk, sc, m_new, nv, full);
                 }
                 if (j > 0) {
                     const bool grow = m_new != m_run;
                     const float alpha = grow ? ex2_approx(m_run - m_new) : 1.0f;
                     if (__any_sync(0xffffffffu, grow)) {
-                        // O must hold tile j-1 before its slice is rescaled
+                        // O must hold tile j-1 before its rows are rescaled; on a
+                        // timeout the rescale is skipped and the next tile's
+                        // barrier takes every slice out
                         const uint32_t tp = tj - 1u;
-                        if (!__all_sync(0xffffffffu,
-                                        mbar_wait(BAR(C::B_PVDONE + (tp & 1u)), (tp >> 1) & 1u, abort_flag))) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
+                        if (__all_sync(0xffffffffu,
+                                       mbar_wait(BAR(C::B_PVDONE + (tp & 1u)), (tp >> 1) & 1u, abort_flag))) {
+                            tc_fence_after();
 #pragma unroll 1
-                        for (int c16 = 0; c16 < OCT / 16; ++c16) {
-                            uint32_t o[16];
-                            const uint32_t ta = tl + (uint32_t)(g * OCT) + 16u * c16;
-                            tmem_ld16(ta, o);
-                            tmem_wait_ld();
+                            for (int c16 = 0; c16 < OCOLS / 16; ++c16) {
+                                uint32_t o[16];
+                                const uint32_t ta = tl + (uint32_t)(h * OCOLS) + 16u * c16;
+                                tmem_ld16(ta, o);
+                                tmem_wait_ld();
 #pragma unroll
-                            for (int e = 0; e < 16; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-                            tmem_st16(ta, o);
+                                for (int e = 0; e < 16; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+                                tmem_st16(ta, o);
+                            }
                         }
-                        tmem_wait_st();
                     }
                     l_part *= alpha;
                 }
                 l_part += rowsum;
                 m_run = m_new;
-                const uint32_t pbase = sP + b * C::PBYTES;
+                // P_j (bf16) into shared buffer b, K-major and 128-byte swizzled as
+                // the A operand of PV_j; the buffer was last read by PV_{j-2}.  On
+                // a timeout the store is skipped and the next barrier takes every
+                // slice out.
+                if (__all_sync(0xffffffffu,
+                               mbar_wait(BAR(C::B_PVDONE + b), ((tj >> 1) & 1u) ^ 1u, abort_flag))) {
+                    const uint32_t pbase = sP + b * C::PBYTES;
 #pragma unroll
-                for (int cc = 0; cc < CPT / 8; ++cc) {
-                    const uint32_t off = sw128_offset(BM, r, g * (CPT / 8) + cc);
-                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(pbase + off), "r"(pk[4 * cc]),
-                                 "r"(pk[4 * cc + 1]), "r"(pk[4 * cc + 2]), "r"(pk[4 * cc + 3]) : "memory");
+                    for (int cc = 0; cc < PCOLS / 4; ++cc) {
+                        const uint32_t off = sw128_offset(BM, r, h * (SCOLS / 8) + cc);
+                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(pbase + off), "r"(pk[4 * cc]),
+                                     "r"(pk[4 * cc + 1]), "r"(pk[4 * cc + 2]), "r"(pk[4 * cc + 3]) : "memory");
+                    }
+                    fence_proxy_async();
                 }
-                fence_proxy_async();
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(BAR(C::B_PFULL + b));
             }
             if (!ok) break;
+            float l_run = 0.f;
             if (n > 0) {
                 const uint32_t tlast = tcnt + (uint32_t)n - 1u;
-                if (!__all_sync(0xffffffffu,
-                                mbar_wait(BAR(C::B_PVDONE + (tlast & 1u)), (tlast >> 1) & 1u, abort_flag))) {
-                    ok = false;
-                    break;
-                }
+                const bool okw = __all_sync(0xffffffffu,
+                                            mbar_wait(BAR(C::B_PVDONE + (tlast & 1u)), (tlast >> 1) & 1u, abort_flag));
+                float *redl = red + (2 * NSPLIT) * BM;
+                redl[h * BM + r] = l_part;
+                if (!bar_and(bar_id, bar_n, okw)) { ok = false; break; }
                 tc_fence_after();
+#pragma unroll
+                for (int q = 0; q < NSPLIT; ++q) l_run += redl[q * BM + r];
             }
             tcnt += (uint32_t)n;
-            // row sum over the groups' slices
-            float l_run = l_part;
-            if (NSM > 1) {
-                red_r[g * BM] = l_part;
-                if (!grp_sync()) { ok = false; break; }
-                l_run = 0.f;
-#pragma unroll
-                for (int q = 0; q < NSM; ++q) l_run += red_r[q * BM];
-                if (!grp_sync()) { ok = false; break; }
-            }
-            // epilogue: this group's O columns [g OCT, (g+1) OCT)
+            // epilogue: this slice's O columns
             const float inv = l_run > 0.f ? 1.0f / l_run : 0.f;
 #pragma unroll 1
-            for (int c16 = 0; c16 < OCT / 16; ++c16) {
+            for (int c16 = 0; c16 < OCOLS / 16; ++c16) {
                 uint32_t o[16];
-                const int col = g * OCT + 16 * c16;
+                const int col = h * OCOLS + 16 * c16;
                 if (n > 0) {
                     tmem_ld16(tl + (uint32_t)col, o);
                     tmem_wait_ld();
@@ -521,13 +488,13 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
                     if (a.residual) {
                         const uint4 *rp = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(a.residual) + off);
 #pragma unroll
-                        for (int q4 = 0; q4 < 2; ++q4) {
-                            const uint4 x = rp[q4];
+                        for (int q4v = 0; q4v < 2; ++q4v) {
+                            const uint4 x = rp[q4v];
                             const uint32_t xw[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
                             for (int e = 0; e < 4; ++e) {
-                                res[8 * q4 + 2 * e] = __uint_as_float(xw[e] << 16);
-                                res[8 * q4 + 2 * e + 1] = __uint_as_float(xw[e] & 0xffff0000u);
+                                res[8 * q4v + 2 * e] = __uint_as_float(xw[e] << 16);
+                                res[8 * q4v + 2 * e + 1] = __uint_as_float(xw[e] & 0xffff0000u);
                             }
                         }
                     } else {
@@ -536,25 +503,25 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
                     }
                     uint4 *dp = reinterpret_cast<uint4 *>(static_cast<uint16_t *>(a.out) + off);
 #pragma unroll
-                    for (int q4 = 0; q4 < 2; ++q4) {
+                    for (int q4v = 0; q4v < 2; ++q4v) {
                         uint32_t pw[4];
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
-                            const int k0 = 8 * q4 + 2 * e;
+                            const int k0 = 8 * q4v + 2 * e;
                             pw[e] = pack_bf16x2(res[k0] + __uint_as_float(o[k0]) * inv,
                                                 res[k0 + 1] + __uint_as_float(o[k0 + 1]) * inv);
                         }
-                        dp[q4] = make_uint4(pw[0], pw[1], pw[2], pw[3]);
+                        dp[q4v] = make_uint4(pw[0], pw[1], pw[2], pw[3]);
                     }
                 } else {
                     float4 *po = reinterpret_cast<float4 *>(a.part_o + ((int64_t)w.slot * BM + r) * DH + col);
 #pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4)
-                        po[q4] = make_float4(__uint_as_float(o[4 * q4]), __uint_as_float(o[4 * q4 + 1]),
-                                             __uint_as_float(o[4 * q4 + 2]), __uint_as_float(o[4 * q4 + 3]));
+                    for (int q4v = 0; q4v < 4; ++q4v)
+                        po[q4v] = make_float4(__uint_as_float(o[4 * q4v]), __uint_as_float(o[4 * q4v + 1]),
+                                              __uint_as_float(o[4 * q4v + 2]), __uint_as_float(o[4 * q4v + 3]));
                 }
             }
-            if (valid && w.slot >= 0 && g == 0)
+            if (valid && w.slot >= 0 && h == 0)
                 reinterpret_cast<float2 *>(a.part_ml)[(int64_t)w.slot * BM + r] = make_float2(m_run, l_run);
             tc_fence_before();
         }

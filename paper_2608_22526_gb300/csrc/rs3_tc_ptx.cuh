@@ -1,5 +1,5 @@
 // rs3_tc_ptx.cuh -- inline-PTX wrappers for the sm_103a tensor-core readout:
-// mbarriers (with bounded waits), TMA tile loads, cp.async, tcgen05 MMA /
+// mbarriers (with bounded waits), TMA tile loads, tcgen05 MMA /
 // commit / TMEM load-store, and the shared-memory and instruction descriptors.
 #pragma once
 
@@ -100,6 +100,8 @@ __device__ __forceinline__ void tc_commit(uint32_t bar)
                  : "memory");
 }
 
+// D (TMEM) [+]= A (shared memory, descriptor) x B (shared memory, descriptor);
+// kind::f16, one CTA.
 __device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
                                        uint32_t accumulate)
 {
@@ -108,6 +110,19 @@ __device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t
         "setp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
         ::"r"(d_tmem), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// D (TMEM) [+]= A (TMEM, K-major: row i in lane i, element pairs per 32-bit
+// column) x B (shared memory, descriptor); kind::f16, one CTA.
+__device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
 
@@ -181,16 +196,6 @@ __device__ __forceinline__ float ex2_approx(float x)
     return y;
 }
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t src_bytes)
-{
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
-}
-
-__device__ __forceinline__ void cp_async_wait_all()
-{
-    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
-}
-
 }  // namespace tc
 
 namespace tc {
@@ -215,6 +220,66 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t *r)
           "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
           "r"(r[15])
         : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t *r)
+{
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                 : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t *r)
+{
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};"
+                 ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]),
+                   "r"(r[7])
+                 : "memory");
+}
+
+// N consecutive 32-bit columns of this warp's 32 lanes (N a multiple of 8).
+template <int N>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t *r)
+{
+    static_assert(N % 8 == 0, "column count");
+    int c = 0;
+#pragma unroll
+    for (; c + 32 <= N; c += 32) tmem_ld32(taddr + (uint32_t)c, r + c);
+    if constexpr (N % 32 >= 16) {
+        tmem_ld16(taddr + (uint32_t)c, r + c);
+        c += 16;
+    }
+    if constexpr (N % 16 == 8) tmem_ld8(taddr + (uint32_t)c, r + c);
+}
+
+template <int N>
+__device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t *r)
+{
+    static_assert(N % 8 == 0, "column count");
+    int c = 0;
+#pragma unroll
+    for (; c + 32 <= N; c += 32) tmem_st32(taddr + (uint32_t)c, r + c);
+    if constexpr (N % 32 >= 16) {
+        tmem_st16(taddr + (uint32_t)c, r + c);
+        c += 16;
+    }
+    if constexpr (N % 16 == 8) tmem_st8(taddr + (uint32_t)c, r + c);
+}
+
+// Named barrier `id` over `nthreads` threads (a multiple of 32) that also
+// ANDs a predicate across them: every participant gets the same answer.
+__device__ __forceinline__ bool bar_and(uint32_t id, uint32_t nthreads, bool pred)
+{
+    uint32_t res;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 q, %1, 0;\n\t"
+        "bar.red.and.pred p, %2, %3, q;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(res)
+        : "r"((uint32_t)pred), "r"(id), "r"(nthreads)
+        : "memory");
+    return res != 0;
 }
 
 }  // namespace tc
