@@ -7,13 +7,14 @@
 // (unit, head, 128-query tile, range of BN-key tiles).  Warps:
 //   warp 0      K producer: TMA of the key tile (d/64 boxes of BN rows x 64)
 //   warp 2      V producer: TMA of the value tile
-//   warp 1      TMEM allocation; one lane issues every MMA:
-//               S_j = Q K_j^T   (M 128, N BN, K d; A = Q in TMEM, B = K tile,
-//                                K-major)
-//               O  += P_j V_j   (M 128, N d, K BN; A = P_j in shared memory,
-//                                B = V tile, MN-major)
-//               S runs two tiles ahead: S_{j+2} is queued as soon as the
-//               softmax has read S_j (two TMEM buffers), before PV_j.
+//   warp 1      TMEM allocation; lane 0 issues S_j = Q K_j^T (M 128, N BN,
+//               K d; A = Q in TMEM, B = K tile, K-major) into one of two TMEM
+//               buffers as soon as the softmax has read the one before
+//   warp 3      lane 0 issues O += P_j V_j (M 128, N d, K BN; A = P_j in
+//               shared memory, B = V tile, MN-major) once P_j is written.  The
+//               two issuers share no operand, so each one's waits overlap the
+//               other's MMAs.
+//   warp 3      lanes 1..31: L2 prefetch of the query rows of later items
 //   warps 4..   2 x 4 softmax warps; warps w and w + 4 own the same TMEM lane
 //               quarter (rows 32 (w % 4) + lane) and split the columns.  Per
 //               item each thread loads its slice of the kept query row,
@@ -21,13 +22,13 @@
 //               writes it to TMEM as bf16 pairs; per tile it reads its slice
 //               of S_j, takes the exps against a running reference that moves
 //               only when the row max grows by more than 2^8 (O is then
-//               rescaled in TMEM), and writes P_j to shared memory (two
+//               rescaled in TMEM), and writes P_j to shared memory (three
 //               buffers).  The slices of a row exchange their maxima through
 //               shared memory at a named barrier that also ANDs their wait
 //               results.  Epilogue: O / l + residual, or split-KV partials.
 // TMEM (512 columns): O in [0, d), S_0 / S_1 from S_COL, Q at Q_COL.
-// Shapes: d = 256 uses 64-key tiles, d = 128 and d = 64 128-key tiles; K and
-// V rings fill what shared memory leaves after the two P buffers.
+// Shapes: d = 256 and d = 128 use 64-key tiles, d = 64 128-key tiles; K and V
+// rings fill what shared memory leaves after the three P buffers.
 // Every mbarrier wait is bounded (1 s of %globaltimer): on expiry the CTA
 // raises an abort flag, drains its copies and MMAs, frees TMEM and the launch
 // latches RS3_ETIMEOUT.
@@ -43,13 +44,14 @@ constexpr uint32_t TMEM_COLS = 512;
 
 template <int DH>
 struct Cfg {
-    static constexpr int BN = DH == 256 ? 64 : 128;          // keys per tile
+    static constexpr int BN = DH == 64 ? 128 : 64;           // keys per tile
     static constexpr int KVBYTES = BN * DH * 2;              // one K (or V) stage
     static constexpr int PBYTES = BM * BN * 2;               // one P buffer
+    static constexpr int NPB = 3;                            // P buffers (and PV barriers)
     static constexpr int NSPLIT = 2;                         // softmax warps per TMEM lane quarter
-    // K stages, V stages: what the 227 KB of shared memory leave after the two
-    // P buffers, the row exchange, the barriers and the alignment slack
-    static constexpr int NKV = (232448 - 1024 - 16 - 64 * 8 - 3 * NSPLIT * BM * 4 - 2 * PBYTES) / KVBYTES;
+    // K stages, V stages: what the 227 KB of shared memory leave after the P
+    // buffers, the row exchange, the barriers and the alignment slack
+    static constexpr int NKV = (232448 - 1024 - 16 - 64 * 8 - 3 * NSPLIT * BM * 4 - NPB * PBYTES) / KVBYTES;
     static constexpr int KSTK = (NKV + 1) / 2, KSTV = NKV / 2;
     static constexpr int NTHREADS = 128 + 128 * NSPLIT;
     static constexpr int SCOLS = BN / NSPLIT;                // S columns of one softmax warp
@@ -61,15 +63,18 @@ struct Cfg {
     static constexpr int OFF_K = 0;
     static constexpr int OFF_V = OFF_K + KSTK * KVBYTES;
     static constexpr int OFF_P = OFF_V + KSTV * KVBYTES;
-    static constexpr int OFF_RED = OFF_P + 2 * PBYTES;       // float [3][NSPLIT][BM]
+    static constexpr int OFF_RED = OFF_P + NPB * PBYTES;     // float [3][NSPLIT][BM]
     static constexpr int OFF_BAR = OFF_RED + 3 * NSPLIT * BM * 4;
-    static constexpr int NBAR = 2 * KSTK + 2 * KSTV + 10;
+    static constexpr int NBAR = 2 * KSTK + 2 * KSTV + 6 + 2 * NPB;
     static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
     static constexpr int SMEM = OFF_MISC + 16 + 1024;        // + alignment slack
     // barrier indices
     static constexpr int B_KFULL = 0, B_KEMPTY = KSTK, B_VFULL = 2 * KSTK, B_VEMPTY = 2 * KSTK + KSTV;
-    static constexpr int B_SFULL = 2 * KSTK + 2 * KSTV, B_SFREE = B_SFULL + 2, B_PFULL = B_SFULL + 4;
-    static constexpr int B_PVDONE = B_SFULL + 6, B_QFULL = B_SFULL + 8, B_DRAIN = B_SFULL + 9;
+    // SFULL / SFREE per S buffer; PFULL / PVDONE per P buffer: the softmax
+    // writes P_{t+3} only after PV_t, so no barrier runs two phases ahead of
+    // its waiter
+    static constexpr int B_SFULL = 2 * KSTK + 2 * KSTV, B_SFREE = B_SFULL + 2, B_QFULL = B_SFULL + 4;
+    static constexpr int B_DRAIN = B_SFULL + 5, B_PFULL = B_SFULL + 6, B_PVDONE = B_PFULL + NPB;
     static_assert(S_COL + 2 * BN <= TMEM_COLS && Q_COL + DH / 2 <= TMEM_COLS, "TMEM budget");
     static_assert(Q_COL >= (uint32_t)DH && (Q_COL + DH / 2 <= S_COL || Q_COL >= S_COL + 2 * BN), "TMEM overlap");
     static_assert(SCOLS % 8 == 0 && PCOLS % 8 == 0 && QCOLS % 8 == 0 && OCOLS % 16 == 0, "warp slices");
@@ -91,55 +96,34 @@ __device__ __forceinline__ float row_max(const uint32_t (&sr)[N], int nv, bool f
     return fmaxf(m0, m1);
 }
 
-// p = 2^(s * sc - ref) packed as bf16 pairs; returns the sum of the p.
+// p = 2^(s * sc - ref) of one slice's scores (raw fp32 bits), as bf16 pairs;
+// returns the sum of the p.  The scale-and-shift and the sums run on packed
+// fp32 pairs (f32x2), the exps on the SFU; four partial sums keep the adds
+// independent.  Columns at or past nv (invalid keys) give p = 0.
 template <int N>
 __device__ __forceinline__ float row_exp(const uint32_t (&sr)[N], uint32_t (&pk)[N / 2], float sc, float ref,
                                          int nv, bool full)
 {
-    const float nref = -ref;
-    float r0 = 0.f, r1 = 0.f;
+    const uint64_t sc2 = f2pack(sc, sc), nref2 = f2pack(-ref, -ref);
+    uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
     for (int c = 0; c < N / 2; ++c) {
-        float p0 = ex2_approx(fmaf(__uint_as_float(sr[2 * c]), sc, nref));
-        float p1 = ex2_approx(fmaf(__uint_as_float(sr[2 * c + 1]), sc, nref));
+        float x0, x1;
+        f2unpack(fma2(f2pack(__uint_as_float(sr[2 * c]), __uint_as_float(sr[2 * c + 1])), sc2, nref2), x0, x1);
+        float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
         if (!full) {
             p0 = 2 * c < nv ? p0 : 0.f;
             p1 = 2 * c + 1 < nv ? p1 : 0.f;
         }
-        r0 += p0;
-        r1 += p1;
+        acc[c & 3] = add2(acc[c & 3], f2pack(p0, p1));
         pk[c] = pack_bf16x2(p0, p1);
     }
-    return r0 + r1;
-}
-
-// row_exp against `ref`, and the max of the valid raw scores in the same pass.
-template <int N>
-__device__ __forceinline__ float row_exp_max(const uint32_t (&sr)[N], uint32_t (&pk)[N / 2], float sc,
-                                             float ref, int nv, bool full, float &mx)
-{
-    const float nref = -ref;
-    float r0 = 0.f, r1 = 0.f, m0 = -INFINITY, m1 = -INFINITY;
-#pragma unroll
-    for (int c = 0; c < N / 2; ++c) {
-        const float s0 = __uint_as_float(sr[2 * c]), s1 = __uint_as_float(sr[2 * c + 1]);
-        float p0 = ex2_approx(fmaf(s0, sc, nref));
-        float p1 = ex2_approx(fmaf(s1, sc, nref));
-        if (full) {
-            m0 = fmaxf(m0, s0);
-            m1 = fmaxf(m1, s1);
-        } else {
-            p0 = 2 * c < nv ? p0 : 0.f;
-            p1 = 2 * c + 1 < nv ? p1 : 0.f;
-            m0 = fmaxf(m0, 2 * c < nv ? s0 : -INFINITY);
-            m1 = fmaxf(m1, 2 * c + 1 < nv ? s1 : -INFINITY);
-        }
-        r0 += p0;
-        r1 += p1;
-        pk[c] = pack_bf16x2(p0, p1);
-    }
-    mx = fmaxf(m0, m1);
-    return r0 + r1;
+    float a0, a1, a2, a3, a4, a5, a6, a7;
+    f2unpack(acc[0], a0, a1);
+    f2unpack(acc[1], a2, a3);
+    f2unpack(acc[2], a4, a5);
+    f2unpack(acc[3], a6, a7);
+    return ((a0 + a1) + (a2 + a3)) + ((a4 + a5) + (a6 + a7));
 }
 
 // NW consecutive bf16 pairs of one thread's kept query row -> its TMEM lane,
@@ -203,11 +187,13 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
         for (int b = 0; b < 2; ++b) {
             mbar_init(BAR(C::B_SFULL + b), 1);
             mbar_init(BAR(C::B_SFREE + b), 4 * C::NSPLIT); // one arrival per softmax warp
+        }
+        for (int b = 0; b < C::NPB; ++b) {
             mbar_init(BAR(C::B_PFULL + b), 4 * C::NSPLIT);
             mbar_init(BAR(C::B_PVDONE + b), 1);
         }
         mbar_init(BAR(C::B_QFULL), 4 * C::NSPLIT);
-        mbar_init(BAR(C::B_DRAIN), 1);
+        mbar_init(BAR(C::B_DRAIN), 2);                    // both MMA issuers
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         fence_proxy_async();
@@ -262,34 +248,16 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             mbar_drain(BAR(b_full + k % nst), (k / nst) & 1u);
     } else if (warp == 1 && lane == 0) {
         // ------------------------------------------------------------------
-        // MMA issuer
+        // S issuer: S_t = Q K_t^T into TMEM buffer t & 1, once the softmax
+        // has read S_{t-2}; runs up to two tiles ahead of the softmax
         // ------------------------------------------------------------------
         constexpr uint32_t ID_S = idesc_bf16(BM, BN, false);
-        constexpr uint32_t ID_PV = idesc_bf16(BM, DH, true);
         // descriptors built once; a k-step only adds its byte offset / 16 to the
         // start-address field (every address stays below 256 KB, so the 14-bit
         // field cannot carry)
-        const uint64_t dk0 = desc_sw128(sK, 16, 1024), dv0 = desc_sw128(sV, BN * 128, 1024);
-        const uint64_t dp0 = desc_sw128(sP, 16, 1024);
-        constexpr uint32_t STAGE16 = C::KVBYTES >> 4, PBUF16 = C::PBYTES >> 4;
+        const uint64_t dk0 = desc_sw128(sK, 16, 1024);
+        constexpr uint32_t STAGE16 = C::KVBYTES >> 4;
         uint32_t tcnt = 0, icnt = 0;
-        // S_t = Q K_t^T into TMEM buffer t & 1, once the softmax has read S_{t-2}
-        auto issue_s = [&](uint32_t t) -> bool {
-            const uint32_t st = t % KSTK, b = t & 1u;
-            if (!mbar_wait(BAR(C::B_SFREE + b), ((t >> 1) & 1u) ^ 1u, abort_flag)) return false;
-            if (!mbar_wait(BAR(C::B_KFULL + st), (t / KSTK) & 1u, abort_flag)) return false;
-            tc_fence_after();
-            const uint64_t dks = dk0 + st * STAGE16;
-            const uint32_t dst = tmem + C::S_COL + (uint32_t)BN * b;
-#pragma unroll
-            for (int kk = 0; kk < DH / 16; ++kk) {
-                const uint32_t offk = (uint32_t)((kk >> 2) * (BN * 128) + (kk & 3) * 32);
-                tc_mma_ts(dst, tmem + C::Q_COL + 8u * kk, dks + (offk >> 4), ID_S, kk > 0 ? 1u : 0u);
-            }
-            tc_commit(BAR(C::B_SFULL + b));
-            tc_commit(BAR(C::B_KEMPTY + st));
-            return true;
-        };
         bool ok = true;
         for (int it = it_begin; it < it_end && ok; ++it) {
             const WorkItem w = a.items[it];
@@ -297,16 +265,43 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             if (n <= 0) continue;
             if (!mbar_wait(BAR(C::B_QFULL), icnt & 1u, abort_flag)) { ok = false; break; }
             ++icnt;
-            tc_fence_after();
-            // S runs two tiles ahead of PV: S_{j+2} is queued before PV_j, so
-            // the softmax of tile j+1 never waits for PV_j
-            if (!issue_s(tcnt)) { ok = false; break; }
-            if (n > 1 && !issue_s(tcnt + 1)) { ok = false; break; }
             for (int j = 0; j < n; ++j) {
-                const uint32_t tj = tcnt + (uint32_t)j, pb = tj & 1u;
-                if (j + 2 < n && !issue_s(tj + 2)) { ok = false; break; }
-                const uint32_t st = tj % KSTV;
-                if (!mbar_wait(BAR(C::B_PFULL + pb), (tj >> 1) & 1u, abort_flag)) { ok = false; break; }
+                const uint32_t t = tcnt + (uint32_t)j, st = t % KSTK, b = t & 1u;
+                if (!mbar_wait(BAR(C::B_SFREE + b), ((t >> 1) & 1u) ^ 1u, abort_flag)) { ok = false; break; }
+                if (!mbar_wait(BAR(C::B_KFULL + st), (t / KSTK) & 1u, abort_flag)) { ok = false; break; }
+                tc_fence_after();
+                const uint64_t dks = dk0 + st * STAGE16;
+                const uint32_t dst = tmem + C::S_COL + (uint32_t)BN * b;
+#pragma unroll
+                for (int kk = 0; kk < DH / 16; ++kk) {
+                    const uint32_t offk = (uint32_t)((kk >> 2) * (BN * 128) + (kk & 3) * 32);
+                    tc_mma_ts(dst, tmem + C::Q_COL + 8u * kk, dks + (offk >> 4), ID_S, kk > 0 ? 1u : 0u);
+                }
+                tc_commit(BAR(C::B_SFULL + b));
+                tc_commit(BAR(C::B_KEMPTY + st));
+            }
+            tcnt += (uint32_t)n;
+        }
+        // every MMA issued by this thread completes before TMEM is released
+        tc_commit(BAR(C::B_DRAIN));
+        mbar_drain(BAR(C::B_DRAIN), 0);
+    } else if (warp == 3 && lane == 0) {
+        // ------------------------------------------------------------------
+        // PV issuer: O += P_t V_t once the softmax has written P_t; its own
+        // thread, so its waits overlap the S issue and the other way round
+        // ------------------------------------------------------------------
+        constexpr uint32_t ID_PV = idesc_bf16(BM, DH, true);
+        const uint64_t dv0 = desc_sw128(sV, BN * 128, 1024), dp0 = desc_sw128(sP, 16, 1024);
+        constexpr uint32_t STAGE16 = C::KVBYTES >> 4, PBUF16 = C::PBYTES >> 4;
+        uint32_t tcnt = 0;
+        bool ok = true;
+        for (int it = it_begin; it < it_end && ok; ++it) {
+            const WorkItem w = a.items[it];
+            const int n = w.tile_end - w.tile_begin;
+            if (n <= 0) continue;
+            for (int j = 0; j < n; ++j) {
+                const uint32_t tj = tcnt + (uint32_t)j, pb = tj % C::NPB, st = tj % KSTV;
+                if (!mbar_wait(BAR(C::B_PFULL + pb), (tj / C::NPB) & 1u, abort_flag)) { ok = false; break; }
                 if (!mbar_wait(BAR(C::B_VFULL + st), (tj / KSTV) & 1u, abort_flag)) { ok = false; break; }
                 tc_fence_after();
                 const uint64_t dvs = dv0 + st * STAGE16, dps = dp0 + pb * PBUF16;
@@ -321,9 +316,32 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             }
             tcnt += (uint32_t)n;
         }
-        // every MMA issued by this thread completes before TMEM is released
         tc_commit(BAR(C::B_DRAIN));
         mbar_drain(BAR(C::B_DRAIN), 0);
+    } else if (warp == 3) {
+        // ------------------------------------------------------------------
+        // lanes 1..31: L2 prefetch of the kept query rows (and their RoPE
+        // rows) of this CTA's later items, so their loads do not wait on DRAM
+        // ------------------------------------------------------------------
+        for (int it = it_begin + 1; it < it_end && !*abort_flag; ++it) {
+            const WorkItem w = a.items[it];
+            if (w.tile_end <= w.tile_begin) continue;
+            const int cnt = __ldg(&a.ranges[w.u].cnt);
+            const int gq = a.unit_group[w.u];
+            for (int rr = lane - 1; rr < BM && w.qt * BM + rr < cnt; rr += 31) {
+                int cell = a.idx[(int64_t)w.u * a.k_max + w.qt * BM + rr];
+                cell = (cell < 0 || cell >= a.mn) ? 0 : cell;
+                const char *qr = reinterpret_cast<const char *>(static_cast<const uint16_t *>(a.q) +
+                                                                ((int64_t)gq * a.mn + cell) * a.D + w.h * DH);
+#pragma unroll
+                for (int l = 0; l < 2 * DH; l += 128) prefetch_l2(qr + l);
+                if (a.rope) {
+                    const char *fr = reinterpret_cast<const char *>(a.rope + (int64_t)cell * DH);
+#pragma unroll
+                    for (int l = 0; l < 4 * DH; l += 128) prefetch_l2(fr + l);
+                }
+            }
+        }
     } else if (warp >= 4) {
         // ------------------------------------------------------------------
         // query rows, softmax / correction, epilogue.  NSPLIT warps share a
@@ -365,19 +383,33 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
                 __syncwarp();
                 if (lane == 0) mbar_arrive(BAR(C::B_QFULL));
             }
+            // the unit's ranges in registers: tile t's valid rows without
+            // global loads in the tile loop
+            int rtiles[4], rlen[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                rtiles[q] = __ldg(&rs->tiles[q]);
+                rlen[q] = __ldg(&rs->len[q]);
+            }
             float m_run = -INFINITY, l_part = 0.f;
             for (int j = 0; j < n; ++j) {
                 const uint32_t tj = tcnt + (uint32_t)j, b = tj & 1u;
                 const bool okw = __all_sync(0xffffffffu, mbar_wait(BAR(C::B_SFULL + b), (tj >> 1) & 1u, abort_flag));
-                int64_t row0;
-                int nvt;
-                tile_rows(rs, w.tile_begin + j, BN, row0, nvt);
+                int nvt = 0;
+                {
+                    int t = w.tile_begin + j;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        if (t >= 0 && t < rtiles[q]) nvt = min(BN, rlen[q] - t * BN);
+                        t -= rtiles[q];
+                    }
+                }
                 const int nv = nvt - h * SCOLS;       // valid columns of this slice (may be <= 0)
                 const bool full = nv >= SCOLS;
                 const uint32_t scol = tl + C::S_COL + (uint32_t)BN * b;
                 const float sc = a.scale_log2;
                 uint32_t sr[SCOLS], pk[PCOLS];
-                float mt, rowsum = 0.f;
+                float rowsum = 0.f;
                 if (okw) {
                     tc_fence_after();
                     tmem_ld_cols<SCOLS>(scol + (uint32_t)(h * SCOLS), sr);
@@ -386,62 +418,74 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(BAR(C::B_SFREE + b));
-                    // After the first tile of an item the exps are taken against
-                    // the running reference m_run, with the slice max gathered in
-                    // the same pass.  The scale is positive, so it is applied to
-                    // the max of the raw scores.
-                    if (j == 0) mt = row_max<SCOLS>(sr, nv, full);
-                    else rowsum = row_exp_max<SCOLS>(sr, pk, sc, m_run, nv, full, mt);
-                } else {
-                    mt = -INFINITY;
                 }
                 float *redt = red + (b * NSPLIT) * BM;
-                redt[h * BM + r] = mt;
-                if (!bar_and(bar_id, bar_n, okw)) { ok = false; break; }
-                float mrow = redt[r];
-#pragma unroll
-                for (int q = 1; q < NSPLIT; ++q) mrow = fmaxf(mrow, redt[q * BM + r]);
-                // the first tile sets the reference; a later one moves it only if
-                // the row max grows past it by more than 2^8 (O is then rescaled)
                 float m_new = m_run;
-                if (j == 0 || mrow * sc > m_run + 8.0f) {
+                if (j == 0) {
+                    // the first tile of an item sets the reference: the row max
+                    // over the slices (the scale is positive, so it is applied
+                    // to the max of the raw scores)
+                    redt[h * BM + r] = okw ? row_max<SCOLS>(sr, nv, full) : -INFINITY;
+                    if (!bar_and(bar_id, bar_n, okw)) { ok = false; break; }
+                    float mrow = redt[r];
+#pragma unroll
+                    for (int q = 1; q < NSPLIT; ++q) mrow = fmaxf(mrow, redt[q * BM + r]);
                     m_new = mrow * sc;
                     rowsum = row_exp<SCOLS>(sr, pk, sc, m_new, nv, full);
-                }
-                if (j > 0) {
-                    const bool grow = m_new != m_run;
-                    const float alpha = grow ? ex2_approx(m_run - m_new) : 1.0f;
-                    if (__any_sync(0xffffffffu, grow)) {
-                        // O must hold tile j-1 before its rows are rescaled; on a
-                        // timeout the rescale is skipped and the next tile's
-                        // barrier takes every slice out
-                        const uint32_t tp = tj - 1u;
-                        if (__all_sync(0xffffffffu,
-                                       mbar_wait(BAR(C::B_PVDONE + (tp & 1u)), (tp >> 1) & 1u, abort_flag))) {
-                            tc_fence_after();
-#pragma unroll 1
-                            for (int c16 = 0; c16 < OCOLS / 16; ++c16) {
-                                uint32_t o[16];
-                                const uint32_t ta = tl + (uint32_t)(h * OCOLS) + 16u * c16;
-                                tmem_ld16(ta, o);
-                                tmem_wait_ld();
+                } else {
+                    // Later tiles take their exps against the running reference.
+                    // It moves only if the row max grows past it by more than
+                    // 2^8, i.e. if some p > 2^8; a row whose sum stays <= 2^8 has
+                    // none, so only rows above that (or a timeout) take the slow
+                    // path, together with their quarter: exact maxima exchanged,
+                    // exps redone against a moved reference, O rescaled.
+                    if (okw) rowsum = row_exp<SCOLS>(sr, pk, sc, m_run, nv, full);
+                    const bool slow = !(rowsum <= 256.0f);
+                    if (bar_or(bar_id, bar_n, slow || !okw)) {
+                        redt[h * BM + r] = okw ? row_max<SCOLS>(sr, nv, full) : -INFINITY;
+                        if (!bar_and(bar_id, bar_n, okw)) { ok = false; break; }
+                        float mrow = redt[r];
 #pragma unroll
-                                for (int e = 0; e < 16; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-                                tmem_st16(ta, o);
+                        for (int q = 1; q < NSPLIT; ++q) mrow = fmaxf(mrow, redt[q * BM + r]);
+                        if (mrow * sc > m_run + 8.0f) {
+                            m_new = mrow * sc;
+                            rowsum = row_exp<SCOLS>(sr, pk, sc, m_new, nv, full);
+                        }
+                        const bool grow = m_new != m_run;
+                        const float alpha = grow ? ex2_approx(m_run - m_new) : 1.0f;
+                        if (__any_sync(0xffffffffu, grow)) {
+                            // O must hold tile j-1 before its rows are rescaled; on
+                            // a timeout the rescale is skipped and the next tile's
+                            // barrier takes every slice out
+                            const uint32_t tp = tj - 1u;
+                            if (__all_sync(0xffffffffu, mbar_wait(BAR(C::B_PVDONE + tp % C::NPB),
+                                                                  (tp / C::NPB) & 1u, abort_flag))) {
+                                tc_fence_after();
+#pragma unroll 1
+                                for (int c16 = 0; c16 < OCOLS / 16; ++c16) {
+                                    uint32_t o[16];
+                                    const uint32_t ta = tl + (uint32_t)(h * OCOLS) + 16u * c16;
+                                    tmem_ld16(ta, o);
+                                    tmem_wait_ld();
+#pragma unroll
+                                    for (int e = 0; e < 16; ++e)
+                                        o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+                                    tmem_st16(ta, o);
+                                }
                             }
                         }
+                        l_part *= alpha;
                     }
-                    l_part *= alpha;
                 }
                 l_part += rowsum;
                 m_run = m_new;
-                // P_j (bf16) into shared buffer b, K-major and 128-byte swizzled as
-                // the A operand of PV_j; the buffer was last read by PV_{j-2}.  On
-                // a timeout the store is skipped and the next barrier takes every
-                // slice out.
-                if (__all_sync(0xffffffffu,
-                               mbar_wait(BAR(C::B_PVDONE + b), ((tj >> 1) & 1u) ^ 1u, abort_flag))) {
-                    const uint32_t pbase = sP + b * C::PBYTES;
+                // P_j (bf16) into shared buffer j % 3, K-major and 128-byte
+                // swizzled as the A operand of PV_j; the buffer was last read by
+                // PV_{j-3}.  On a timeout the store is skipped and the next
+                // barrier takes every slice out.
+                if (__all_sync(0xffffffffu, mbar_wait(BAR(C::B_PVDONE + tj % C::NPB),
+                                                      ((tj / C::NPB) & 1u) ^ 1u, abort_flag))) {
+                    const uint32_t pbase = sP + (tj % C::NPB) * C::PBYTES;
 #pragma unroll
                     for (int cc = 0; cc < PCOLS / 4; ++cc) {
                         const uint32_t off = sw128_offset(BM, r, h * (SCOLS / 8) + cc);
@@ -452,14 +496,14 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
                 }
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(BAR(C::B_PFULL + b));
+                if (lane == 0) mbar_arrive(BAR(C::B_PFULL + tj % C::NPB));
             }
             if (!ok) break;
             float l_run = 0.f;
             if (n > 0) {
                 const uint32_t tlast = tcnt + (uint32_t)n - 1u;
-                const bool okw = __all_sync(0xffffffffu,
-                                            mbar_wait(BAR(C::B_PVDONE + (tlast & 1u)), (tlast >> 1) & 1u, abort_flag));
+                const bool okw = __all_sync(0xffffffffu, mbar_wait(BAR(C::B_PVDONE + tlast % C::NPB),
+                                                                   (tlast / C::NPB) & 1u, abort_flag));
                 float *redl = red + (2 * NSPLIT) * BM;
                 redl[h * BM + r] = l_part;
                 if (!bar_and(bar_id, bar_n, okw)) { ok = false; break; }
@@ -468,57 +512,52 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
                 for (int q = 0; q < NSPLIT; ++q) l_run += redl[q * BM + r];
             }
             tcnt += (uint32_t)n;
-            // epilogue: this slice's O columns
+            // epilogue: this slice's O columns, EG chunks of 16 at a time with
+            // their residual loads issued together
             const float inv = l_run > 0.f ? 1.0f / l_run : 0.f;
+            constexpr int EG = OCOLS >= 32 ? 2 : 1;
 #pragma unroll 1
-            for (int c16 = 0; c16 < OCOLS / 16; ++c16) {
-                uint32_t o[16];
-                const int col = h * OCOLS + 16 * c16;
+            for (int c0 = 0; c0 < OCOLS; c0 += 16 * EG) {
+                const int col0 = h * OCOLS + c0;
+                const int64_t off = ((int64_t)w.u * a.mn + cell) * a.D + w.h * DH + col0;
+                uint4 res[2 * EG];
+                if (valid && w.slot < 0) {
+#pragma unroll
+                    for (int q = 0; q < 2 * EG; ++q)
+                        res[q] = a.residual ? __ldg(reinterpret_cast<const uint4 *>(
+                                                  static_cast<const uint16_t *>(a.residual) + off) + q)
+                                            : make_uint4(0u, 0u, 0u, 0u);
+                }
+                uint32_t o[16 * EG];
                 if (n > 0) {
-                    tmem_ld16(tl + (uint32_t)col, o);
+#pragma unroll
+                    for (int e = 0; e < EG; ++e) tmem_ld16(tl + (uint32_t)(col0 + 16 * e), o + 16 * e);
                     tmem_wait_ld();
                 } else {
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) o[e] = 0u;
+                    for (int e = 0; e < 16 * EG; ++e) o[e] = 0u;
                 }
                 if (!valid) continue;
                 if (w.slot < 0) {
-                    const int64_t off = ((int64_t)w.u * a.mn + cell) * a.D + w.h * DH + col;
-                    float res[16];
-                    if (a.residual) {
-                        const uint4 *rp = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(a.residual) + off);
-#pragma unroll
-                        for (int q4v = 0; q4v < 2; ++q4v) {
-                            const uint4 x = rp[q4v];
-                            const uint32_t xw[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                res[8 * q4v + 2 * e] = __uint_as_float(xw[e] << 16);
-                                res[8 * q4v + 2 * e + 1] = __uint_as_float(xw[e] & 0xffff0000u);
-                            }
-                        }
-                    } else {
-#pragma unroll
-                        for (int e = 0; e < 16; ++e) res[e] = 0.f;
-                    }
                     uint4 *dp = reinterpret_cast<uint4 *>(static_cast<uint16_t *>(a.out) + off);
 #pragma unroll
-                    for (int q4v = 0; q4v < 2; ++q4v) {
+                    for (int q = 0; q < 2 * EG; ++q) {
+                        const uint32_t xw[4] = {res[q].x, res[q].y, res[q].z, res[q].w};
                         uint32_t pw[4];
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
-                            const int k0 = 8 * q4v + 2 * e;
-                            pw[e] = pack_bf16x2(res[k0] + __uint_as_float(o[k0]) * inv,
-                                                res[k0 + 1] + __uint_as_float(o[k0 + 1]) * inv);
+                            const int k0 = 8 * q + 2 * e;
+                            pw[e] = pack_bf16x2(__uint_as_float(xw[e] << 16) + __uint_as_float(o[k0]) * inv,
+                                                __uint_as_float(xw[e] & 0xffff0000u) + __uint_as_float(o[k0 + 1]) * inv);
                         }
-                        dp[q4v] = make_uint4(pw[0], pw[1], pw[2], pw[3]);
+                        dp[q] = make_uint4(pw[0], pw[1], pw[2], pw[3]);
                     }
                 } else {
-                    float4 *po = reinterpret_cast<float4 *>(a.part_o + ((int64_t)w.slot * BM + r) * DH + col);
+                    float4 *po = reinterpret_cast<float4 *>(a.part_o + ((int64_t)w.slot * BM + r) * DH + col0);
 #pragma unroll
-                    for (int q4v = 0; q4v < 4; ++q4v)
-                        po[q4v] = make_float4(__uint_as_float(o[4 * q4v]), __uint_as_float(o[4 * q4v + 1]),
-                                              __uint_as_float(o[4 * q4v + 2]), __uint_as_float(o[4 * q4v + 3]));
+                    for (int q = 0; q < 4 * EG; ++q)
+                        __stcg(po + q, make_float4(__uint_as_float(o[4 * q]), __uint_as_float(o[4 * q + 1]),
+                                                   __uint_as_float(o[4 * q + 2]), __uint_as_float(o[4 * q + 3])));
                 }
             }
             if (valid && w.slot >= 0 && h == 0)

@@ -78,6 +78,11 @@ __device__ __forceinline__ void mbar_drain(uint32_t bar, uint32_t parity)
         if (gtimer() - t0 > WAIT_LIMIT_NS) return;
 }
 
+__device__ __forceinline__ void prefetch_l2(const void *p)
+{
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 __device__ __forceinline__ void fence_proxy_async()
 {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -264,6 +269,50 @@ __device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t *r)
         c += 16;
     }
     if constexpr (N % 16 == 8) tmem_st8(taddr + (uint32_t)c, r + c);
+}
+
+// Named barrier `id` over `nthreads` threads (a multiple of 32) that also
+// ORs a predicate across them: every participant gets the same answer.
+__device__ __forceinline__ bool bar_or(uint32_t id, uint32_t nthreads, bool pred)
+{
+    uint32_t res;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 q, %1, 0;\n\t"
+        "bar.red.or.pred p, %2, %3, q;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(res)
+        : "r"((uint32_t)pred), "r"(id), "r"(nthreads)
+        : "memory");
+    return res != 0;
+}
+
+// Packed fp32 pairs (sm_100+ f32x2 arithmetic): two lanes of work per
+// instruction, each rounded exactly as the scalar operation.
+__device__ __forceinline__ uint64_t f2pack(float lo, float hi)
+{
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+
+__device__ __forceinline__ void f2unpack(uint64_t v, float &lo, float &hi)
+{
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c)
+{
+    uint64_t d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b)
+{
+    uint64_t d;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
 }
 
 // Named barrier `id` over `nthreads` threads (a multiple of 32) that also
