@@ -148,7 +148,7 @@ class DeviceSequence:
         import torch
         from paper_2608_22526_gb300 import synth
         seq = synth.Sequence(w)
-        T = w.frames
+        T = w.frames + w.prefill_frames           # sequence frames, prefill first
         ug = w.unit_group()
         esz = 2 if w.dtype == "bf16" else 4
         per_frame = (w.G + 3 * w.U) * w.mn * w.D * esz
@@ -180,6 +180,7 @@ class DeviceSequence:
         self.dev = {k: v.to(device) for k, v in self.host.items()}
         self.masks_np = masks
         self.T = T
+        self.P = w.prefill_frames
 
     def frame(self, key, t):
         """Device tensor of input `key` for frame t."""
@@ -245,9 +246,12 @@ def run_step(pipe, data, timers=None, side=None):
         if timers is not None:
             sel_t[t][1] = ev
 
-    first = 1 if w.n_cond > 0 else 0
+    first = data.P + (1 if w.n_cond > 0 else 0)
     for t in range(data.T):
-        if t == 0 and w.n_cond > 0:
+        if t < data.P:                       # unpruned frames already in the bank
+            pipe.commit(F("k", t), F("v", t), None, 0)
+            continue
+        if t == data.P and w.n_cond > 0:
             pipe.commit(F("k", t), F("v", t), F("mask", t), 1)
             if data.ptr is not None:
                 pipe.set_pointers(*data.ptr)
@@ -295,7 +299,10 @@ def work_model(pipe, data):
     pipe.track.zero_()
     out = []
     for t in range(data.T):
-        if t == 0 and w.n_cond > 0:
+        if t < data.P:
+            pipe.commit(F("k", t), F("v", t), None, 0)
+            continue
+        if t == data.P and w.n_cond > 0:
             pipe.commit(F("k", t), F("v", t), F("mask", t), 1)
             if data.ptr is not None:
                 pipe.set_pointers(*data.ptr)
@@ -451,8 +458,8 @@ def gpu_arm(args):
         "mean_queries": round(float(np.mean([sum(c) for c in P["counts"]])), 1),
         "mean_bank_rows": round(float(np.mean([sum(n) for n in P["lens"]])), 1),
         "clocks": P["clocks"],
-        "gpu_launches": (1 + (2 if w.n_ptr > 0 else 1) + (w.frames - (1 if w.n_cond > 0 else 0))
-                         * KERNELS_PER_READOUT_FRAME) * args.steps,
+        "gpu_launches": (1 + w.prefill_frames + (2 if w.n_ptr > 0 else 1)
+                         + (w.frames - (1 if w.n_cond > 0 else 0)) * KERNELS_PER_READOUT_FRAME) * args.steps,
     }
     if "dense" in results:
         Dn = results["dense"]
