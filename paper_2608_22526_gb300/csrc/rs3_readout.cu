@@ -256,6 +256,7 @@ __global__ void __launch_bounds__(1024) k_plan(ReadoutArgs a)
         hdr->n_items = (int32_t)ri;
         hdr->n_combine = (int32_t)rc;
         hdr->pad[0] = v.P;
+        hdr->pad[1] = (int32_t)rp;                  // partial pieces of all split groups
     }
 }
 
@@ -392,20 +393,75 @@ __global__ void __launch_bounds__(512) k_readout_simt(ReadoutArgs a)
 // ---------------------------------------------------------------------------
 // k_combine: log-sum-exp merge of split-KV partials, then the scatter
 // ---------------------------------------------------------------------------
-template <typename T>
+// A warp takes one output row: the row's splits' (m, l) pairs give M = max m
+// and L = sum 2^(m - M) l; each lane accumulates E columns per CW-column chunk
+// over the splits with weight 2^(m_s - M) (eight splits' loads in flight at a
+// time) and stores residual + sum / L.  When the groups are split many ways
+// (small frames spread over all SMs) a row is shared by one warp per chunk;
+// otherwise one warp does the whole row (lanes striding the columns four at a
+// time), so the loads of the row's entry, cell and (m, l) pairs are not
+// repeated per chunk.
+template <typename T, int E>
+__device__ __forceinline__ void store_out_e(const ReadoutArgs &a, int u, int cell, int c, const float *o);
+
+template <>
+__device__ __forceinline__ void store_out_e<float, 1>(const ReadoutArgs &a, int u, int cell, int c, const float *o)
+{
+    const int64_t off = ((int64_t)u * a.mn + cell) * a.D + c;
+    const float r = a.residual ? static_cast<const float *>(a.residual)[off] : 0.f;
+    static_cast<float *>(a.out)[off] = r + o[0];
+}
+
+template <>
+__device__ __forceinline__ void store_out_e<float, 2>(const ReadoutArgs &a, int u, int cell, int c, const float *o)
+{
+    const int64_t off = ((int64_t)u * a.mn + cell) * a.D + c;
+    float2 r = make_float2(0.f, 0.f);
+    if (a.residual) r = *reinterpret_cast<const float2 *>(static_cast<const float *>(a.residual) + off);
+    *reinterpret_cast<float2 *>(static_cast<float *>(a.out) + off) = make_float2(r.x + o[0], r.y + o[1]);
+}
+
+template <>
+__device__ __forceinline__ void store_out_e<uint16_t, 1>(const ReadoutArgs &a, int u, int cell, int c, const float *o)
+{
+    const int64_t off = ((int64_t)u * a.mn + cell) * a.D + c;
+    const float r = a.residual ? bf16_bits_to_float(static_cast<const uint16_t *>(a.residual)[off]) : 0.f;
+    static_cast<uint16_t *>(a.out)[off] = float_to_bf16_bits(r + o[0]);
+}
+
+template <>
+__device__ __forceinline__ void store_out_e<uint16_t, 2>(const ReadoutArgs &a, int u, int cell, int c, const float *o)
+{
+    const int64_t off = ((int64_t)u * a.mn + cell) * a.D + c;
+    float r0 = 0.f, r1 = 0.f;
+    if (a.residual) {
+        const uint32_t x = *reinterpret_cast<const uint32_t *>(static_cast<const uint16_t *>(a.residual) + off);
+        r0 = __uint_as_float(x << 16);
+        r1 = __uint_as_float(x & 0xffff0000u);
+    }
+    *reinterpret_cast<uint32_t *>(static_cast<uint16_t *>(a.out) + off) = pack_bf16x2(r0 + o[0], r1 + o[1]);
+}
+
+template <typename T, int E>
 __global__ void __launch_bounds__(256) k_combine(ReadoutArgs a)
 {
-    // one warp per output row: lane s holds split s's (m, l); lanes then
-    // stride the columns, every split's partial loaded without waiting on the
-    // previous one
-    const int64_t n_rows = (int64_t)a.header->n_combine * a.BM;
-    const int lane = threadIdx.x & 31;
+    constexpr int CW = 32 * E;                      // columns per warp
     const int d = a.d;
+    // chunked tasks only when the groups are split more than four ways on
+    // average (one decision for the launch, so no task is spent idle)
+    const int n_comb = a.header->n_combine;
+    const bool chunked = a.header->pad[1] > 4 * n_comb;
+    const int chunks = chunked ? (d + CW - 1) / CW : 1;   // tasks per row
+    const int64_t n_tasks = (int64_t)n_comb * a.BM * chunks;
+    const int lane = threadIdx.x & 31;
     const float2 *pm = reinterpret_cast<const float2 *>(a.part_ml);
-    for (int64_t gr = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; gr < n_rows;
-         gr += ((int64_t)gridDim.x * blockDim.x) >> 5) {
+    for (int64_t task = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; task < n_tasks;
+         task += ((int64_t)gridDim.x * blockDim.x) >> 5) {
+        const int64_t gr = task / chunks;
+        const int chunk = (int)(task % chunks);
         const int ci = (int)(gr / a.BM), r = (int)(gr % a.BM);
         const CombineItem c = a.combine[ci];
+        const bool whole = !chunked;
         const int j = c.qt * a.BM + r;
         if (j >= a.ranges[c.u].cnt) continue;          // warp-uniform
         int cell = a.idx[(int64_t)c.u * a.k_max + j];
@@ -424,21 +480,45 @@ __global__ void __launch_bounds__(256) k_combine(ReadoutArgs a)
         L = warp_sum(L);
         const float inv = L > 0.f ? 1.f / L : 0.f;
         const int64_t sstride = (int64_t)a.BM * d;
-        for (int c4 = lane * 4; c4 < d; c4 += 128) {              // no warp collectives below
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            const float *base = a.part_o + ((int64_t)c.slot0 * a.BM + r) * d + c4;
+        if (whole) {
+            // lanes stride the row's columns four at a time; no warp collectives
+            for (int c4 = lane * 4; c4 < d; c4 += 128) {
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                const float *base = a.part_o + ((int64_t)c.slot0 * a.BM + r) * d + c4;
 #pragma unroll 4
-            for (int s = 0; s < c.nsplit; ++s) {
-                const float ws = M == -INFINITY ? 0.f : exp2f(ml[(int64_t)s * a.BM].x - M);
-                const float4 po = __ldcs(reinterpret_cast<const float4 *>(base + s * sstride));
-                acc.x = fmaf(ws, po.x, acc.x);
-                acc.y = fmaf(ws, po.y, acc.y);
-                acc.z = fmaf(ws, po.z, acc.z);
-                acc.w = fmaf(ws, po.w, acc.w);
+                for (int s = 0; s < c.nsplit; ++s) {
+                    const float ws = M == -INFINITY ? 0.f : exp2f(ml[(int64_t)s * a.BM].x - M);
+                    const float4 po = __ldcs(reinterpret_cast<const float4 *>(base + s * sstride));
+                    acc.x = fmaf(ws, po.x, acc.x);
+                    acc.y = fmaf(ws, po.y, acc.y);
+                    acc.z = fmaf(ws, po.z, acc.z);
+                    acc.w = fmaf(ws, po.w, acc.w);
+                }
+                const float o4[4] = {acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv};
+                store_out4<T>(a, c.u, cell, c.h * d + c4, o4);
             }
-            float o4[4] = {acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv};
-            store_out4<T>(a, c.u, cell, c.h * d + c4, o4);
+            continue;
         }
+        const int col = chunk * CW + lane * E;
+        if (col >= d) continue;                          // d < 32 only; no collectives below
+        const float *base = a.part_o + ((int64_t)c.slot0 * a.BM + r) * d + col;
+        float acc[E];
+#pragma unroll
+        for (int e = 0; e < E; ++e) acc[e] = 0.f;
+#pragma unroll 8
+        for (int s = 0; s < c.nsplit; ++s) {
+            const float ws = M == -INFINITY ? 0.f : exp2f(ml[(int64_t)s * a.BM].x - M);
+            if constexpr (E == 2) {
+                const float2 po = __ldcs(reinterpret_cast<const float2 *>(base + s * sstride));
+                acc[0] = fmaf(ws, po.x, acc[0]);
+                acc[1] = fmaf(ws, po.y, acc[1]);
+            } else {
+                acc[0] = fmaf(ws, __ldcs(base + s * sstride), acc[0]);
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < E; ++e) acc[e] *= inv;
+        store_out_e<T, E>(a, c.u, cell, c.h * d + col, acc);
     }
 }
 
@@ -618,14 +698,20 @@ rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_
             k_readout_simt<float><<<(unsigned)blocks, threads, smem, st>>>(a);
         if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     }
-    int64_t cblocks = (max_combine * a.BM + 7) / 8;     // one warp per partial row
-    const int64_t ccap = (int64_t)a.n_sm * 8;
+    // one warp per (partial row, 64-column chunk; 32 for d < 64)
+    const int ce = a.d >= 64 ? 2 : 1;
+    const int64_t chunks = (a.d + 32 * ce - 1) / (32 * ce);
+    int64_t cblocks = (max_combine * a.BM * chunks + 7) / 8;
+    const int64_t ccap = (int64_t)a.n_sm * 16;
     if (cblocks > ccap) cblocks = ccap;
     if (cblocks < 1) cblocks = 1;
-    if (dtype == RS3_BF16)
-        k_combine<uint16_t><<<(unsigned)cblocks, 256, 0, st>>>(a);
-    else
-        k_combine<float><<<(unsigned)cblocks, 256, 0, st>>>(a);
+    if (dtype == RS3_BF16) {
+        if (ce == 2) k_combine<uint16_t, 2><<<(unsigned)cblocks, 256, 0, st>>>(a);
+        else k_combine<uint16_t, 1><<<(unsigned)cblocks, 256, 0, st>>>(a);
+    } else {
+        if (ce == 2) k_combine<float, 2><<<(unsigned)cblocks, 256, 0, st>>>(a);
+        else k_combine<float, 1><<<(unsigned)cblocks, 256, 0, st>>>(a);
+    }
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     return RS3_OK;
 }

@@ -79,6 +79,8 @@ struct Cfg {
     static_assert(Q_COL >= (uint32_t)DH && (Q_COL + DH / 2 <= S_COL || Q_COL >= S_COL + 2 * BN), "TMEM overlap");
     static_assert(SCOLS % 8 == 0 && PCOLS % 8 == 0 && QCOLS % 8 == 0 && OCOLS % 16 == 0, "warp slices");
     static_assert(KSTK >= 2 && KSTV >= 2 && NBAR <= 64, "K/V stages");
+    static_assert(4 * NSPLIT * 32 * 36 * 4 <= NPB * PBYTES, "epilogue staging fits in the P ring");
+    static_assert(OCOLS % 32 == 0, "epilogue stages 32 columns at a time");
 };
 static_assert(Cfg<256>::SMEM <= 232448 && Cfg<128>::SMEM <= 232448 && Cfg<64>::SMEM <= 232448,
               "shared memory budget");
@@ -512,33 +514,66 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
                 for (int q = 0; q < NSPLIT; ++q) l_run += redl[q * BM + r];
             }
             tcnt += (uint32_t)n;
-            // epilogue: this slice's O columns, EG chunks of 16 at a time with
-            // their residual loads issued together
             const float inv = l_run > 0.f ? 1.0f / l_run : 0.f;
-            constexpr int EG = OCOLS >= 32 ? 2 : 1;
+            if (w.slot >= 0) {
+                // split-KV partial (fp32, unnormalised): 32 columns at a time are
+                // staged through shared memory so that each store instruction
+                // writes four whole rows of 128 bytes.  The staging area is this
+                // warp's part of the P ring, idle from the item's last PV (waited
+                // for above) until the next item's first P, which no warp writes
+                // before every warp has passed this epilogue (QFULL).
+                float *stg = reinterpret_cast<float *>(gbase + C::OFF_P) + (warp - 4) * (32 * 36);
+                float *pdst = a.part_o + ((int64_t)w.slot * BM + 32 * q4) * DH + h * OCOLS;
 #pragma unroll 1
-            for (int c0 = 0; c0 < OCOLS; c0 += 16 * EG) {
-                const int col0 = h * OCOLS + c0;
-                const int64_t off = ((int64_t)w.u * a.mn + cell) * a.D + w.h * DH + col0;
-                uint4 res[2 * EG];
-                if (valid && w.slot < 0) {
+                for (int c0 = 0; c0 < OCOLS; c0 += 32) {
+                    uint32_t o[32];
+                    if (n > 0) {
+                        tmem_ld32(tl + (uint32_t)(h * OCOLS + c0), o);
+                        tmem_wait_ld();
+                    } else {
 #pragma unroll
-                    for (int q = 0; q < 2 * EG; ++q)
-                        res[q] = a.residual ? __ldg(reinterpret_cast<const uint4 *>(
-                                                  static_cast<const uint16_t *>(a.residual) + off) + q)
-                                            : make_uint4(0u, 0u, 0u, 0u);
+                        for (int e = 0; e < 32; ++e) o[e] = 0u;
+                    }
+                    __syncwarp();
+#pragma unroll
+                    for (int k = 0; k < 8; ++k)
+                        *reinterpret_cast<uint4 *>(stg + lane * 36 + 4 * k) =
+                            make_uint4(o[4 * k], o[4 * k + 1], o[4 * k + 2], o[4 * k + 3]);
+                    __syncwarp();
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) {
+                        const int row = 4 * q + (lane >> 3), c4 = 4 * (lane & 7);
+                        __stcg(reinterpret_cast<float4 *>(pdst + (int64_t)row * DH + c0 + c4),
+                               *reinterpret_cast<const float4 *>(stg + row * 36 + c4));
+                    }
                 }
-                uint32_t o[16 * EG];
-                if (n > 0) {
+            } else {
+                // out = residual + O / l at the kept cell, rounded once to bf16;
+                // EG chunks of 16 columns at a time with their residual loads
+                // issued together
+                constexpr int EG = OCOLS >= 32 ? 2 : 1;
+#pragma unroll 1
+                for (int c0 = 0; c0 < OCOLS; c0 += 16 * EG) {
+                    const int col0 = h * OCOLS + c0;
+                    const int64_t off = ((int64_t)w.u * a.mn + cell) * a.D + w.h * DH + col0;
+                    uint4 res[2 * EG];
+                    if (valid) {
 #pragma unroll
-                    for (int e = 0; e < EG; ++e) tmem_ld16(tl + (uint32_t)(col0 + 16 * e), o + 16 * e);
-                    tmem_wait_ld();
-                } else {
+                        for (int q = 0; q < 2 * EG; ++q)
+                            res[q] = a.residual ? __ldg(reinterpret_cast<const uint4 *>(
+                                                      static_cast<const uint16_t *>(a.residual) + off) + q)
+                                                : make_uint4(0u, 0u, 0u, 0u);
+                    }
+                    uint32_t o[16 * EG];
+                    if (n > 0) {
 #pragma unroll
-                    for (int e = 0; e < 16 * EG; ++e) o[e] = 0u;
-                }
-                if (!valid) continue;
-                if (w.slot < 0) {
+                        for (int e = 0; e < EG; ++e) tmem_ld16(tl + (uint32_t)(col0 + 16 * e), o + 16 * e);
+                        tmem_wait_ld();
+                    } else {
+#pragma unroll
+                        for (int e = 0; e < 16 * EG; ++e) o[e] = 0u;
+                    }
+                    if (!valid) continue;
                     uint4 *dp = reinterpret_cast<uint4 *>(static_cast<uint16_t *>(a.out) + off);
 #pragma unroll
                     for (int q = 0; q < 2 * EG; ++q) {
@@ -552,12 +587,6 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
                         }
                         dp[q] = make_uint4(pw[0], pw[1], pw[2], pw[3]);
                     }
-                } else {
-                    float4 *po = reinterpret_cast<float4 *>(a.part_o + ((int64_t)w.slot * BM + r) * DH + col0);
-#pragma unroll
-                    for (int q = 0; q < 4 * EG; ++q)
-                        __stcg(po + q, make_float4(__uint_as_float(o[4 * q]), __uint_as_float(o[4 * q + 1]),
-                                                   __uint_as_float(o[4 * q + 2]), __uint_as_float(o[4 * q + 3])));
                 }
             }
             if (valid && w.slot >= 0 && h == 0)
