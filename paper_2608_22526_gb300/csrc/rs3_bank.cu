@@ -66,6 +66,7 @@ k_commit(const uint8_t *__restrict__ k_new, const uint8_t *__restrict__ v_new,
          const uint8_t *__restrict__ mask, int mn, int is_cond, int64_t row_bytes, BankDev bk,
          uint8_t *__restrict__ k_store, uint8_t *__restrict__ v_store, int32_t *status)
 {
+    pdl_wait();
     __shared__ int32_t s_list[COMMIT_CHUNK];
     __shared__ int32_t s_red[2][8];
     __shared__ int s_last;
@@ -200,6 +201,7 @@ __global__ void k_set_pointers(const uint8_t *__restrict__ kp, const uint8_t *__
                                int64_t row_bytes, BankDev bk, uint8_t *__restrict__ k_store,
                                uint8_t *__restrict__ v_store)
 {
+    pdl_wait();
     const int u = blockIdx.x;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
     const int nvec = (int)(row_bytes / 16);
@@ -217,6 +219,7 @@ __global__ void k_set_pointers(const uint8_t *__restrict__ kp, const uint8_t *__
 
 __global__ void k_bank_reset(BankDev bk, int unit, int U)
 {
+    pdl_wait();
     const int u0 = unit < 0 ? 0 : unit, u1 = unit < 0 ? U : unit + 1;
     for (int u = u0 + blockIdx.x; u < u1; u += gridDim.x) {
         int64_t *mu = bk.meta + (int64_t)u * bk.stride_words;
@@ -299,7 +302,7 @@ extern "C" rs3_status rs3_bank_commit(const rs3_bank *bank, const void *k_new, c
     const int mn = bank->mn;
     const int nchunks = (mn + COMMIT_CHUNK - 1) / COMMIT_CHUNK;
     const int64_t row_bytes = (int64_t)bank->D * (int64_t)elem_bytes(bank->dtype);
-    k_commit<<<dim3(nchunks, bank->U), 256, 0, st>>>(
+    launch_pdl(k_commit, dim3(nchunks, bank->U), dim3(256), 0, st,
         static_cast<const uint8_t *>(k_new), static_cast<const uint8_t *>(v_new), keep_mask, mn, is_cond,
         row_bytes, bk, static_cast<uint8_t *>(bank->k_store), static_cast<uint8_t *>(bank->v_store), status);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
@@ -313,7 +316,7 @@ extern "C" rs3_status rs3_bank_set_pointers(const rs3_bank *bank, const void *k_
     if (bank->n_ptr == 0) return RS3_EINVAL;
     if (!rs3_aligned16(k_ptr) || !rs3_aligned16(v_ptr)) return RS3_EINVAL;
     const int64_t row_bytes = (int64_t)bank->D * (int64_t)elem_bytes(bank->dtype);
-    k_set_pointers<<<bank->U, 256, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+    launch_pdl(k_set_pointers, dim3(bank->U), dim3(256), 0, reinterpret_cast<cudaStream_t>(stream),
         static_cast<const uint8_t *>(k_ptr), static_cast<const uint8_t *>(v_ptr), row_bytes,
         bank_dev(bank), static_cast<uint8_t *>(bank->k_store), static_cast<uint8_t *>(bank->v_store));
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
@@ -325,7 +328,7 @@ extern "C" rs3_status rs3_bank_reset(const rs3_bank *bank, int unit, rs3_stream_
     if (!bank_ok(bank)) return RS3_EINVAL;
     if (unit < -1 || unit >= bank->U) return RS3_EINVAL;
     const int blocks = unit < 0 ? (bank->U < 1024 ? bank->U : 1024) : 1;
-    k_bank_reset<<<blocks, 32, 0, reinterpret_cast<cudaStream_t>(stream)>>>(bank_dev(bank), unit,
+    launch_pdl(k_bank_reset, dim3(blocks), dim3(32), 0, reinterpret_cast<cudaStream_t>(stream), bank_dev(bank), unit,
                                                                             bank->U);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     return RS3_OK;

@@ -104,6 +104,35 @@ __device__ __forceinline__ T warp_sum(T v)
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// ---------------------------------------------------------------------------
+// Programmatic dependent launch.  Every kernel of the library is launched with
+// programmatic stream serialisation, so its launch is processed while the
+// previous kernel of its stream runs; pdl_wait() returns once that kernel has
+// completed and its writes are visible (at once when there is none), and every
+// kernel calls it before its first global-memory access.  No kernel triggers
+// its dependents early: they are scheduled when it completes, so kernels
+// waiting for their predecessor never hold SMs that the selection running on
+// another stream could use.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                              Args &&...args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
+
 // Host helpers implemented in rs3_api.cu
 int rs3_sm_count();
 bool rs3_aligned16(const void *p);

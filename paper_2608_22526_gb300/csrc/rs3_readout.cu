@@ -27,6 +27,7 @@ namespace {
 // ---------------------------------------------------------------------------
 __global__ void k_passthrough(const uint4 *__restrict__ res, uint4 *__restrict__ out, int64_t nvec)
 {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nvec;
          i += (int64_t)gridDim.x * blockDim.x)
         out[i] = res ? __ldcs(res + i) : make_uint4(0, 0, 0, 0);
@@ -178,6 +179,7 @@ __device__ void plan_slice(const ReadoutArgs &a, const PlanView &v, int b, bool 
 
 __global__ void __launch_bounds__(1024) k_plan(ReadoutArgs a)
 {
+    pdl_wait();
     ReadoutHeader *hdr = a.header;
     extern __shared__ int64_t s_plan[];            // [U+1] tb, [U] wg, [3][grid+1] per-CTA counts
     int64_t *s_tb = s_plan, *s_wg = s_plan + (a.U + 1);
@@ -272,6 +274,7 @@ constexpr int SIMT_BN = 32;
 template <typename T>
 __global__ void __launch_bounds__(512) k_readout_simt(ReadoutArgs a)
 {
+    pdl_wait();
     extern __shared__ __align__(16) float sm[];
     const int d = a.d;
     const int TPR = d / 16;
@@ -445,6 +448,7 @@ __device__ __forceinline__ void store_out_e<uint16_t, 2>(const ReadoutArgs &a, i
 template <typename T, int E>
 __global__ void __launch_bounds__(256) k_combine(ReadoutArgs a)
 {
+    pdl_wait();
     constexpr int CW = 32 * E;                      // columns per warp
     const int d = a.d;
     // chunked tasks only when the groups are split more than four ways on
@@ -662,7 +666,7 @@ rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_
         int64_t blocks = (nvec + 255) / 256;
         const int64_t cap = (int64_t)a.n_sm * 8;
         if (blocks > cap) blocks = cap;
-        k_passthrough<<<(unsigned)blocks, 256, 0, st>>>(static_cast<const uint4 *>(a.residual),
+        launch_pdl(k_passthrough, dim3((unsigned)blocks), dim3(256), 0, st, static_cast<const uint4 *>(a.residual),
                                                         static_cast<uint4 *>(a.out), nvec);
         if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     }
@@ -675,7 +679,7 @@ rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_
             return RS3_EUNSUPPORTED;
         plan_attr = plan_smem;
     }
-    k_plan<<<1, 1024, plan_smem, st>>>(a);
+    launch_pdl(k_plan, dim3(1), dim3(1024), plan_smem, st, a);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     (void)max_items;
     if (p.kind == 1) {
@@ -693,9 +697,9 @@ rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_
             attr_done = true;
         }
         if (dtype == RS3_BF16)
-            k_readout_simt<uint16_t><<<(unsigned)blocks, threads, smem, st>>>(a);
+            launch_pdl(k_readout_simt<uint16_t>, dim3((unsigned)blocks), dim3(threads), smem, st, a);
         else
-            k_readout_simt<float><<<(unsigned)blocks, threads, smem, st>>>(a);
+            launch_pdl(k_readout_simt<float>, dim3((unsigned)blocks), dim3(threads), smem, st, a);
         if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     }
     // one warp per (partial row, 64-column chunk; 32 for d < 64)
@@ -706,11 +710,11 @@ rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_
     if (cblocks > ccap) cblocks = ccap;
     if (cblocks < 1) cblocks = 1;
     if (dtype == RS3_BF16) {
-        if (ce == 2) k_combine<uint16_t, 2><<<(unsigned)cblocks, 256, 0, st>>>(a);
-        else k_combine<uint16_t, 1><<<(unsigned)cblocks, 256, 0, st>>>(a);
+        if (ce == 2) launch_pdl(k_combine<uint16_t, 2>, dim3((unsigned)cblocks), dim3(256), 0, st, a);
+        else launch_pdl(k_combine<uint16_t, 1>, dim3((unsigned)cblocks), dim3(256), 0, st, a);
     } else {
-        if (ce == 2) k_combine<float, 2><<<(unsigned)cblocks, 256, 0, st>>>(a);
-        else k_combine<float, 1><<<(unsigned)cblocks, 256, 0, st>>>(a);
+        if (ce == 2) launch_pdl(k_combine<float, 2>, dim3((unsigned)cblocks), dim3(256), 0, st, a);
+        else launch_pdl(k_combine<float, 1>, dim3((unsigned)cblocks), dim3(256), 0, st, a);
     }
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     return RS3_OK;

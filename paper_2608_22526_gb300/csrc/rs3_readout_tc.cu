@@ -213,6 +213,9 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // the set-up above touches no global memory; the plan is read after the
+    // previous kernel of the stream has completed
+    pdl_wait();
     // this CTA's slice of the stream-K plan
     const int it_begin = a.cta_items[blockIdx.x], it_end = a.cta_items[blockIdx.x + 1];
 
@@ -652,7 +655,7 @@ rs3_status launch(const ReadoutArgs &a, cudaStream_t st)
         !make_kv_map(&mv, a.v_store, a.D, rows, Cfg<DH>::BN))
         return RS3_ECUDA;
     const int64_t grid = a.grid_ctas;               // the plan's slices; unused ones exit at once
-    k_readout_tc<DH><<<(unsigned)grid, Cfg<DH>::NTHREADS, Cfg<DH>::SMEM, st>>>(a, mk, mv);
+    launch_pdl(k_readout_tc<DH>, dim3((unsigned)grid), dim3(Cfg<DH>::NTHREADS), Cfg<DH>::SMEM, st, a, mk, mv);
     return cudaGetLastError() == cudaSuccess ? RS3_OK : RS3_ECUDA;
 }
 

@@ -98,6 +98,7 @@ k_prior(const uint8_t *__restrict__ masks, int m, int n, const int32_t *__restri
         int G, rs3_track *__restrict__ track, int r_s, int c, int bbox_mode,
         uint8_t *__restrict__ prior, uint32_t *__restrict__ need, int32_t *status)
 {
+    pdl_wait();
     extern __shared__ __align__(16) uint8_t smem[];
     const int mn = m * n;
     const int u = blockIdx.x;
@@ -210,6 +211,7 @@ __global__ void __launch_bounds__(256)
 k_energy(const T *__restrict__ z, int G, int mn, int C, int lpr, const uint32_t *__restrict__ need,
          float *__restrict__ e)
 {
+    pdl_wait();
     const int nchunk = C >> 3;
     const int rpw = 32 / lpr;
     const int lane = threadIdx.x & 31;
@@ -277,6 +279,7 @@ k_select(const uint8_t *__restrict__ prior, const uint32_t *__restrict__ need,
          const float *__restrict__ e, const int32_t *__restrict__ unit_group, int G, int mn,
          int union_mode, int k, int32_t *__restrict__ idx, int32_t *__restrict__ count)
 {
+    pdl_wait();
     extern __shared__ __align__(16) uint32_t skey[];
     __shared__ uint32_t hist[256];
     __shared__ uint32_t s_bin, s_rem;
@@ -386,6 +389,7 @@ k_write_keepset(const uint8_t *__restrict__ seeds, const int32_t *__restrict__ u
                 int G_unused, int m, int n, int D_w, double fall_lo, double fall_hi,
                 int fall_through, int union_mode, uint8_t *__restrict__ kw, int32_t *status)
 {
+    pdl_wait();
     extern __shared__ __align__(16) uint8_t smem[];
     const int mn = m * n;
     const int u = blockIdx.x;
@@ -479,7 +483,7 @@ extern "C" rs3_status rs3_select_queries(const void *z, rs3_dtype dtype, int G, 
 
     if (cudaMemsetAsync(need, 0, (size_t)G * nwords * 4, st) != cudaSuccess) return RS3_ECUDA;
     const size_t smem_prior = 2 * (size_t)((mn + 15) & ~15);
-    k_prior<<<U, 1024, smem_prior, st>>>(prev_masks, m, n, unit_group, G, track, p->r_s, p->c,
+    launch_pdl(k_prior, dim3(U), dim3(1024), smem_prior, st, prev_masks, m, n, unit_group, G, track, p->r_s, p->c,
                                          p->bbox_mode, prior, need, status);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
 
@@ -493,10 +497,10 @@ extern "C" rs3_status rs3_select_queries(const void *z, rs3_dtype dtype, int G, 
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
     if (dtype == RS3_BF16)
-        k_energy<uint16_t><<<(unsigned)blocks, 256, 0, st>>>(static_cast<const uint16_t *>(z), G, mn, C,
+        launch_pdl(k_energy<uint16_t>, dim3((unsigned)blocks), dim3(256), 0, st, static_cast<const uint16_t *>(z), G, mn, C,
                                                            lpr, need, energy);
     else
-        k_energy<float><<<(unsigned)blocks, 256, 0, st>>>(static_cast<const float *>(z), G, mn, C, lpr,
+        launch_pdl(k_energy<float>, dim3((unsigned)blocks), dim3(256), 0, st, static_cast<const float *>(z), G, mn, C, lpr,
                                                         need, energy);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
 
@@ -506,7 +510,7 @@ extern "C" rs3_status rs3_select_queries(const void *z, rs3_dtype dtype, int G, 
         cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, RS3_MAX_MN * 4);
         attr_set = true;
     }
-    k_select<<<U, 1024, smem_sel, st>>>(prior, need, energy, unit_group, G, mn, p->union_mode,
+    launch_pdl(k_select, dim3(U), dim3(1024), smem_sel, st, prior, need, energy, unit_group, G, mn, p->union_mode,
                                         (int)k, idx, count);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     return RS3_OK;
@@ -522,7 +526,7 @@ extern "C" rs3_status rs3_write_keepset(const uint8_t *seed_masks, const int32_t
     const int mn = m * n;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const size_t smem = 2 * (size_t)((mn + 15) & ~15);
-    k_write_keepset<<<U, 1024, smem, st>>>(seed_masks, unit_group, U, 0, m, n, p->D_w, p->fall_lo,
+    launch_pdl(k_write_keepset, dim3(U), dim3(1024), smem, st, seed_masks, unit_group, U, 0, m, n, p->D_w, p->fall_lo,
                                            p->fall_hi, p->fall_through, p->union_mode, kw_out,
                                            status);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
