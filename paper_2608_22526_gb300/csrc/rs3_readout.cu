@@ -102,22 +102,19 @@ __device__ int64_t block_scan64(int64_t v, int64_t *total)
 // Stream-K plan.  Group g = (unit u, query tile qt, head h) owns
 // wg_u = max(T_u, 1) consecutive slots of a linear work axis (T_u = key tiles
 // of the unit's bank; an empty bank keeps one slot so its rows are written).
-// CTA b of P takes slots [b W / P, (b+1) W / P) and its slice is cut at group
-// boundaries into items.  A group that a slice boundary cuts is split: its
-// pieces write partials to consecutive slots (CTA order) and the CTA holding
-// its first piece emits the combine entry.
+// CTA b of P takes slots [sb[b], sb[b+1]) with sb[b] = b W / P, and its slice
+// is cut at group boundaries into items.  A group that a slice boundary cuts
+// is split: its pieces write partials to consecutive slots (CTA order) and the
+// CTA holding its first piece emits the combine entry.
 struct PlanView {
     const int64_t *tb;   // [U+1] first linear slot of each unit
     const int64_t *wg;   // [U]   slots per group of each unit
+    const int32_t *nt;   // [U]   key tiles of each unit
+    const int64_t *sb;   // [P+1] first slot of each slice
     int U, H;
     int64_t W;
     int P;
 };
-
-__device__ __forceinline__ int64_t slice_begin(const PlanView &v, int b)
-{
-    return (int64_t)b * v.W / v.P;
-}
 
 __device__ __forceinline__ void locate(const PlanView &v, int64_t x, int &u, int &gl, int64_t &off)
 {
@@ -138,7 +135,7 @@ __device__ void plan_slice(const ReadoutArgs &a, const PlanView &v, int b, bool 
                            int64_t slot0, int64_t comb0, int &n_items, int &n_part, int &n_comb)
 {
     n_items = n_part = n_comb = 0;
-    const int64_t lo = slice_begin(v, b), hi = slice_begin(v, b + 1);
+    const int64_t lo = v.sb[b], hi = v.sb[b + 1];
     for (int64_t x = lo; x < hi;) {
         int u, gl;
         int64_t off;
@@ -147,23 +144,27 @@ __device__ void plan_slice(const ReadoutArgs &a, const PlanView &v, int b, bool 
         const int64_t len = min(hi - x, wg - off);
         const bool whole = off == 0 && len == wg;
         if (write) {
-            const RangeSet &rs = a.ranges[u];
+            const int64_t nt = v.nt[u];
             WorkItem w;
             w.u = u; w.qt = gl / v.H; w.h = gl % v.H; w.split = 0;
-            w.tile_begin = (int32_t)min(off, (int64_t)rs.n_tiles);
-            w.tile_end = (int32_t)min(off + len, (int64_t)rs.n_tiles);
+            w.tile_begin = (int32_t)min(off, nt);
+            w.tile_end = (int32_t)min(off + len, nt);
             w.slot = whole ? -1 : (int32_t)(slot0 + n_part);
             w.pad = 0;
             a.items[item0 + n_items] = w;
             if (!whole && off == 0) {
-                // first piece of a split group: count the slices it spans
-                const int64_t gend = x + wg - 1;            // last slot of the group
-                int e = b;
-                while (e + 1 < v.P && slice_begin(v, e + 1) <= gend) ++e;
+                // first piece of a split group: the last slice it reaches is the
+                // last e with sb[e] <= its last slot
+                const int64_t gend = x + wg - 1;
+                int lo_e = b, hi_e = v.P;                  // sb[lo_e] <= gend < sb[hi_e]
+                while (hi_e - lo_e > 1) {
+                    const int mid = (lo_e + hi_e) >> 1;
+                    if (v.sb[mid] <= gend) lo_e = mid; else hi_e = mid;
+                }
                 CombineItem c;
                 c.u = u; c.h = w.h; c.qt = w.qt;
                 c.slot0 = (int32_t)(slot0 + n_part);
-                c.nsplit = e - b + 1;
+                c.nsplit = lo_e - b + 1;
                 c.pad[0] = c.pad[1] = c.pad[2] = 0;
                 a.combine[comb0 + n_comb] = c;
             }
@@ -177,13 +178,22 @@ __device__ void plan_slice(const ReadoutArgs &a, const PlanView &v, int b, bool 
     }
 }
 
-__global__ void __launch_bounds__(1024) k_plan(ReadoutArgs a)
+// Per-CTA counts packed in one int64 for a single scan: items in bits 0..20,
+// partial pieces in 21..41, combine entries in 42..62 (every total is far
+// below 2^21: items <= groups + CTAs).
+constexpr int PK_SHIFT = 21;
+constexpr int64_t PK_MASK = (1ll << PK_SHIFT) - 1;
+
+constexpr int PLAN_THREADS = 256;
+
+__global__ void __launch_bounds__(PLAN_THREADS) k_plan(ReadoutArgs a)
 {
     pdl_wait();
     ReadoutHeader *hdr = a.header;
-    extern __shared__ int64_t s_plan[];            // [U+1] tb, [U] wg, [3][grid+1] per-CTA counts
-    int64_t *s_tb = s_plan, *s_wg = s_plan + (a.U + 1);
-    int64_t *s_ci = s_wg + a.U, *s_cp = s_ci + (a.grid_ctas + 1), *s_cc = s_cp + (a.grid_ctas + 1);
+    // [U+1] tb, [U] wg, [grid+1] sb, [grid+1] packed per-CTA counts, [U] nt (int32)
+    extern __shared__ int64_t s_plan[];
+    int64_t *s_tb = s_plan, *s_wg = s_tb + (a.U + 1), *s_sb = s_wg + a.U, *s_pk = s_sb + (a.grid_ctas + 1);
+    int32_t *s_nt = reinterpret_cast<int32_t *>(s_pk + (a.grid_ctas + 1));
     for (int u = threadIdx.x; u < a.U; u += blockDim.x) {
         int cnt = a.count[u];
         if (cnt < 0 || cnt > a.k_max) {
@@ -210,50 +220,53 @@ __global__ void __launch_bounds__(1024) k_plan(ReadoutArgs a)
         }
         a.ranges[u] = rs;
         s_wg[u] = rs.n_tiles > 0 ? rs.n_tiles : 1;
+        s_nt[u] = rs.n_tiles;
+        s_tb[u] = (int64_t)rs.nq * a.H * s_wg[u];   // this unit's slots, scanned below
     }
     __syncthreads();
     // linear slot base of every unit (exclusive scan in rounds of blockDim)
     int64_t run = 0;
     for (int u0 = 0; u0 < a.U; u0 += blockDim.x) {
         const int u = u0 + threadIdx.x;
-        const int64_t w = u < a.U ? (int64_t)a.ranges[u].nq * a.H * s_wg[u] : 0;
+        const int64_t w = u < a.U ? s_tb[u] : 0;
         int64_t tot;
         const int64_t off = block_scan64(w, &tot) + run;
         if (u < a.U) s_tb[u] = off;
         run += tot;
     }
     if (threadIdx.x == 0) s_tb[a.U] = run;
-    __syncthreads();
-    PlanView v;
-    v.tb = s_tb; v.wg = s_wg; v.U = a.U; v.H = a.H; v.W = run;
     int64_t P = (run + a.min_chunk - 1) / a.min_chunk;
     if (P > a.grid_ctas) P = a.grid_ctas;
+    for (int b = threadIdx.x; b <= P; b += blockDim.x) s_sb[b] = P > 0 ? (int64_t)b * run / P : 0;
+    __syncthreads();
+    PlanView v;
+    v.tb = s_tb; v.wg = s_wg; v.nt = s_nt; v.sb = s_sb; v.U = a.U; v.H = a.H; v.W = run;
     v.P = (int)P;
-    // per-CTA counts, then exclusive scans into offsets
+    // per-CTA counts, then one exclusive scan into offsets
     for (int b = threadIdx.x; b < v.P; b += blockDim.x) {
         int ni, np, nc;
         plan_slice(a, v, b, false, 0, 0, 0, ni, np, nc);
-        s_ci[b] = ni; s_cp[b] = np; s_cc[b] = nc;
+        s_pk[b] = (int64_t)ni | ((int64_t)np << PK_SHIFT) | ((int64_t)nc << (2 * PK_SHIFT));
     }
     __syncthreads();
-    int64_t ri = 0, rp = 0, rc = 0;
+    int64_t rsum = 0;
     for (int b0 = 0; b0 < v.P; b0 += blockDim.x) {
         const int b = b0 + threadIdx.x;
-        const int64_t ni = b < v.P ? s_ci[b] : 0, np = b < v.P ? s_cp[b] : 0, nc = b < v.P ? s_cc[b] : 0;
-        int64_t ti, tp, tc;
-        const int64_t oi = block_scan64(ni, &ti) + ri;
-        const int64_t op = block_scan64(np, &tp) + rp;
-        const int64_t oc = block_scan64(nc, &tc) + rc;
-        if (b < v.P) { s_ci[b] = oi; s_cp[b] = op; s_cc[b] = oc; }
-        ri += ti; rp += tp; rc += tc;
+        int64_t tot;
+        const int64_t off = block_scan64(b < v.P ? s_pk[b] : 0, &tot) + rsum;
+        if (b < v.P) s_pk[b] = off;
+        rsum += tot;
     }
     __syncthreads();
     for (int b = threadIdx.x; b < v.P; b += blockDim.x) {
         int ni, np, nc;
-        plan_slice(a, v, b, true, s_ci[b], s_cp[b], s_cc[b], ni, np, nc);
+        const int64_t o = s_pk[b];
+        plan_slice(a, v, b, true, o & PK_MASK, (o >> PK_SHIFT) & PK_MASK, (o >> (2 * PK_SHIFT)) & PK_MASK, ni,
+                   np, nc);
     }
+    const int64_t ri = rsum & PK_MASK, rp = (rsum >> PK_SHIFT) & PK_MASK, rc = (rsum >> (2 * PK_SHIFT)) & PK_MASK;
     for (int b = threadIdx.x; b <= a.grid_ctas; b += blockDim.x)
-        a.cta_items[b] = (int32_t)(b < v.P ? s_ci[b] : ri);
+        a.cta_items[b] = (int32_t)(b < v.P ? (s_pk[b] & PK_MASK) : ri);
     if (threadIdx.x == 0) {
         hdr->n_items = (int32_t)ri;
         hdr->n_combine = (int32_t)rc;
@@ -671,7 +684,7 @@ rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_
         if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     }
     // plan shared memory: unit slot bases and widths, per-CTA counts
-    const size_t plan_smem = ((size_t)(2 * a.U + 1) + 3 * (size_t)(a.grid_ctas + 1)) * 8;
+    const size_t plan_smem = ((size_t)(2 * a.U + 1) + 2 * (size_t)(a.grid_ctas + 1)) * 8 + (size_t)a.U * 4;
     static size_t plan_attr = 0;
     if (plan_smem > 48 * 1024 && plan_smem > plan_attr) {
         if (cudaFuncSetAttribute(k_plan, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan_smem) !=
@@ -679,7 +692,7 @@ rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_
             return RS3_EUNSUPPORTED;
         plan_attr = plan_smem;
     }
-    launch_pdl(k_plan, dim3(1), dim3(1024), plan_smem, st, a);
+    launch_pdl(k_plan, dim3(1), dim3(PLAN_THREADS), plan_smem, st, a);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     (void)max_items;
     if (p.kind == 1) {
