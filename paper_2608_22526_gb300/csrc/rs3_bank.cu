@@ -57,8 +57,8 @@ __device__ __forceinline__ int nonzero_bytes(uint4 w)
 // [c * COMMIT_CHUNK, (c+1) * COMMIT_CHUNK) of unit u.  Every CTA reads the
 // unit's old counters, counts the unit's kept rows (and those before its
 // chunk), takes the same eviction / capacity decision, ranks its kept cells
-// with ballot/popc and copies their K and V rows with 128-bit loads and
-// stores, a warp per row.  The last CTA of the unit to finish (an arrival
+// with ballot/popc and copies their K and V rows as 16-byte pieces spread
+// over all its threads.  The last CTA of the unit to finish (an arrival
 // count in the unit's metadata, after a fence) publishes the new counters and
 // the frame-table entry, so no CTA can see counters of the frame it copies.
 __global__ void __launch_bounds__(256)
@@ -68,6 +68,7 @@ k_commit(const uint8_t *__restrict__ k_new, const uint8_t *__restrict__ v_new,
 {
     pdl_wait();
     __shared__ int32_t s_list[COMMIT_CHUNK];
+    __shared__ int64_t s_row[COMMIT_CHUNK];
     __shared__ int32_t s_red[2][8];
     __shared__ int s_last;
     const int u = blockIdx.y, ch = blockIdx.x;
@@ -147,22 +148,41 @@ k_commit(const uint8_t *__restrict__ k_new, const uint8_t *__restrict__ v_new,
         if (keep) {
             uint32_t lm;
             asm("mov.u32 %0, %%lanemask_lt;" : "=r"(lm));
-            s_list[off + __popc(bal & lm)] = cell;
+            const int j = off + __popc(bal & lm);
+            const int64_t rank = pre + j;
+            s_list[j] = cell;
+            s_row[j] = is_cond ? base + rank : bk.pinned_cap + (base + rank) % bk.ring_cap;
         }
         __syncthreads();
+        // the chunk's rows as 16-byte pieces over all threads, four pieces'
+        // K and V loads in flight before their stores
         const int nvec = (int)(row_bytes / 16);
+        const int npiece = nk * nvec;
         const uint8_t *ksrc = k_new + (size_t)u * mn * row_bytes;
         const uint8_t *vsrc = v_new + (size_t)u * mn * row_bytes;
         uint8_t *kdst = k_store + (size_t)u * bk.rows_per_unit * row_bytes;
         uint8_t *vdst = v_store + (size_t)u * bk.rows_per_unit * row_bytes;
-        for (int j = warp; j < nk; j += 8) {
-            const int64_t rank = pre + j;
-            const int64_t row = is_cond ? base + rank : bk.pinned_cap + (base + rank) % bk.ring_cap;
-            const int64_t c = s_list[j];
-            copy_row(reinterpret_cast<uint4 *>(kdst + row * row_bytes),
-                     reinterpret_cast<uint4 *>(vdst + row * row_bytes),
-                     reinterpret_cast<const uint4 *>(ksrc + c * row_bytes),
-                     reinterpret_cast<const uint4 *>(vsrc + c * row_bytes), nvec, lane);
+        for (int i0 = threadIdx.x; i0 < npiece; i0 += 4 * blockDim.x) {
+            uint4 kk[4], vv[4];
+            int64_t dst[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int i = i0 + q * blockDim.x;
+                if (i < npiece) {
+                    const int j = i / nvec, v = i - j * nvec;
+                    const int64_t so = (int64_t)s_list[j] * row_bytes + 16 * v;
+                    dst[q] = s_row[j] * row_bytes + 16 * v;
+                    kk[q] = __ldcs(reinterpret_cast<const uint4 *>(ksrc + so));
+                    vv[q] = __ldcs(reinterpret_cast<const uint4 *>(vsrc + so));
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                if (i0 + q * (int)blockDim.x < npiece) {
+                    *reinterpret_cast<uint4 *>(kdst + dst[q]) = kk[q];
+                    *reinterpret_cast<uint4 *>(vdst + dst[q]) = vv[q];
+                }
+            }
         }
     }
 
