@@ -100,12 +100,16 @@ __device__ int64_t block_scan64(int64_t v, int64_t *total)
 }
 
 // Stream-K plan.  Group g = (unit u, query tile qt, head h) owns
-// wg_u = max(T_u, 1) consecutive slots of a linear work axis (T_u = key tiles
-// of the unit's bank; an empty bank keeps one slot so its rows are written).
-// CTA b of P takes slots [sb[b], sb[b+1]) with sb[b] = b W / P, and its slice
-// is cut at group boundaries into items.  A group that a slice boundary cuts
-// is split: its pieces write partials to consecutive slots (CTA order) and the
-// CTA holding its first piece emits the combine entry.
+// wg_u = OV + T_u consecutive slots of a linear work axis (T_u = key tiles of
+// the unit's bank): OV leading slots stand for the fixed cost of starting a
+// piece of work (loading the query rows, the epilogue), so a CTA whose slice
+// starts groups gets fewer tiles, and the T_u tile slots follow.  CTA b of P
+// takes slots [sb[b], sb[b+1]) with sb[b] = b W / P; its slice is cut at group
+// boundaries into items, each the tiles of the group its part covers.  A group
+// whose tiles a slice boundary cuts is split: its pieces write partials to
+// consecutive slots (CTA order) and the CTA holding its first tile emits the
+// combine entry.  A group with no tiles (empty bank) is one item with no
+// tiles, emitted where its first slot lies, so its rows are still written.
 struct PlanView {
     const int64_t *tb;   // [U+1] first linear slot of each unit
     const int64_t *wg;   // [U]   slots per group of each unit
@@ -114,6 +118,7 @@ struct PlanView {
     int U, H;
     int64_t W;
     int P;
+    int ov;              // leading slots of a group (the start-up cost)
 };
 
 __device__ __forceinline__ void locate(const PlanView &v, int64_t x, int &u, int &gl, int64_t &off)
@@ -142,37 +147,43 @@ __device__ void plan_slice(const ReadoutArgs &a, const PlanView &v, int b, bool 
         locate(v, x, u, gl, off);
         const int64_t wg = v.wg[u];
         const int64_t len = min(hi - x, wg - off);
-        const bool whole = off == 0 && len == wg;
-        if (write) {
-            const int64_t nt = v.nt[u];
-            WorkItem w;
-            w.u = u; w.qt = gl / v.H; w.h = gl % v.H; w.split = 0;
-            w.tile_begin = (int32_t)min(off, nt);
-            w.tile_end = (int32_t)min(off + len, nt);
-            w.slot = whole ? -1 : (int32_t)(slot0 + n_part);
-            w.pad = 0;
-            a.items[item0 + n_items] = w;
-            if (!whole && off == 0) {
-                // first piece of a split group: the last slice it reaches is the
-                // last e with sb[e] <= its last slot
-                const int64_t gend = x + wg - 1;
-                int lo_e = b, hi_e = v.P;                  // sb[lo_e] <= gend < sb[hi_e]
-                while (hi_e - lo_e > 1) {
-                    const int mid = (lo_e + hi_e) >> 1;
-                    if (v.sb[mid] <= gend) lo_e = mid; else hi_e = mid;
+        const int64_t nt = v.nt[u];
+        // the tiles this part covers, and whether it holds all or the first
+        const int64_t t0 = min(max(off - v.ov, (int64_t)0), nt);
+        const int64_t t1 = min(max(off + len - v.ov, (int64_t)0), nt);
+        const bool emit = nt > 0 ? t1 > t0 : off == 0;
+        if (emit) {
+            const bool whole = t0 == 0 && t1 == nt;
+            if (write) {
+                WorkItem w;
+                w.u = u; w.qt = gl / v.H; w.h = gl % v.H; w.split = 0;
+                w.tile_begin = (int32_t)t0;
+                w.tile_end = (int32_t)t1;
+                w.slot = whole ? -1 : (int32_t)(slot0 + n_part);
+                w.pad = 0;
+                a.items[item0 + n_items] = w;
+                if (!whole && t0 == 0) {
+                    // first piece of a split group: the last slice it reaches is
+                    // the last e with sb[e] <= the group's last slot
+                    const int64_t gend = x - off + wg - 1;
+                    int lo_e = b, hi_e = v.P;              // sb[lo_e] <= gend < sb[hi_e]
+                    while (hi_e - lo_e > 1) {
+                        const int mid = (lo_e + hi_e) >> 1;
+                        if (v.sb[mid] <= gend) lo_e = mid; else hi_e = mid;
+                    }
+                    CombineItem c;
+                    c.u = u; c.h = w.h; c.qt = w.qt;
+                    c.slot0 = (int32_t)(slot0 + n_part);
+                    c.nsplit = lo_e - b + 1;
+                    c.pad[0] = c.pad[1] = c.pad[2] = 0;
+                    a.combine[comb0 + n_comb] = c;
                 }
-                CombineItem c;
-                c.u = u; c.h = w.h; c.qt = w.qt;
-                c.slot0 = (int32_t)(slot0 + n_part);
-                c.nsplit = lo_e - b + 1;
-                c.pad[0] = c.pad[1] = c.pad[2] = 0;
-                a.combine[comb0 + n_comb] = c;
             }
-        }
-        ++n_items;
-        if (!whole) {
-            if (off == 0) ++n_comb;
-            ++n_part;
+            ++n_items;
+            if (!whole) {
+                if (t0 == 0) ++n_comb;
+                ++n_part;
+            }
         }
         x += len;
     }
@@ -219,7 +230,7 @@ __global__ void __launch_bounds__(PLAN_THREADS) k_plan(ReadoutArgs a)
             rs = unit_ranges(a, u, cnt);
         }
         a.ranges[u] = rs;
-        s_wg[u] = rs.n_tiles > 0 ? rs.n_tiles : 1;
+        s_wg[u] = (int64_t)a.plan_ov + rs.n_tiles;
         s_nt[u] = rs.n_tiles;
         s_tb[u] = (int64_t)rs.nq * a.H * s_wg[u];   // this unit's slots, scanned below
     }
@@ -241,6 +252,7 @@ __global__ void __launch_bounds__(PLAN_THREADS) k_plan(ReadoutArgs a)
     __syncthreads();
     PlanView v;
     v.tb = s_tb; v.wg = s_wg; v.nt = s_nt; v.sb = s_sb; v.U = a.U; v.H = a.H; v.W = run;
+    v.ov = a.plan_ov;
     v.P = (int)P;
     // per-CTA counts, then one exclusive scan into offsets
     for (int b = threadIdx.x; b < v.P; b += blockDim.x) {
@@ -653,6 +665,9 @@ rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, in
     a->BN = p.BN;
     a->n_sm = rs3_sm_count();
     a->min_chunk = p.kind == 1 ? 2 : 4;
+    // start-up cost of a piece in tile slots: the tensor-core path's query
+    // load and epilogue take about as long as four 64-key tiles
+    a->plan_ov = p.kind == 1 ? 4 : 1;
     a->max_slots = L.max_slots;
     a->max_items = L.max_items;
     a->grid_ctas = p.grid;

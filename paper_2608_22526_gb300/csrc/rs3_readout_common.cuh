@@ -23,6 +23,7 @@ struct ReadoutArgs {
     int32_t *status;
     int U, G, mn, H, d, D, k_max;
     int BM, BN, n_sm, min_chunk;
+    int plan_ov;            // leading plan slots per group: a piece's start-up cost in tiles
     int64_t max_slots;
     int64_t max_items;
     int grid_ctas;          // CTAs of the readout launch (the plan's slice count bound)
