@@ -665,9 +665,9 @@ rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, in
     a->BN = p.BN;
     a->n_sm = rs3_sm_count();
     a->min_chunk = p.kind == 1 ? 2 : 4;
-    // start-up cost of a piece in tile slots: the tensor-core path's query
-    // load and epilogue take about as long as four 64-key tiles
-    a->plan_ov = p.kind == 1 ? 4 : 1;
+    // start-up cost of a piece in tile slots: on the tensor-core path a
+    // sweep of 4..32 over the 1- and 8-object sequences was best at 8..16
+    a->plan_ov = p.kind == 1 ? 12 : 1;
     a->max_slots = L.max_slots;
     a->max_items = L.max_items;
     a->grid_ctas = p.grid;
