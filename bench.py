@@ -206,21 +206,28 @@ class DeviceSequence:
 
 
 OVERLAP = "readout"
+SPLIT_MERGE = True
 
 
-def run_step(pipe, data, timers=None, side=None):
+def run_step(pipe, data, timers=None, side=None, merge=None):
     """One step: the whole sequence through the library (Algorithm 1's loop).
 
     The selection of frame t+1 needs only frame t+1's grid and frame t's mask,
     so it is issued on `side`: with OVERLAP == "commit" it runs beside frame
     t's commit (after frame t's readout, so the persistent readout always has
     every SM), with "readout" beside the readout and commit, with "none" in
-    line on the main stream."""
+    line on the main stream.  With SPLIT_MERGE the readout runs as its two
+    phases: the attention on the main stream, the split-KV merge on `merge`
+    beside the frame's commit (the merge reads no bank); the next attention
+    waits for the merge, which shares its workspace."""
     import torch
     w = pipe.w
     from paper_2608_22526_gb300 import rs3
     main = torch.cuda.current_stream()
     side = side if (side is not None and OVERLAP != "none") else main
+    # the per-call timing pass (timers) keeps each frame's calls back to back
+    # on one stream, so that their event times are the calls' own durations
+    mrg = merge if (merge is not None and SPLIT_MERGE and timers is None) else main
     rs3.rs3_bank_reset(pipe.bank, -1)
     pipe.track.zero_()
     F = data.frame
@@ -261,24 +268,35 @@ def run_step(pipe, data, timers=None, side=None):
         if t + 1 < data.T and OVERLAP == "readout":
             issue_select(t + 1)          # beside this frame's readout and commit
         main.wait_event(sel_ev[t])
+        if t - 1 in rd_ev and mrg is not main:
+            main.wait_event(rd_ev[t - 1])   # the previous merge still reads the workspace
         pipe.use_buffer(t % 2)
         if timers is not None:
-            e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
             e[0].record(main)
-        pipe.readout(F("z", t), F("x", t), F("x", t))
+        pipe.readout_attend(F("z", t), F("x", t), F("x", t))
+        att = torch.cuda.Event(enable_timing=timers is not None)
+        att.record(main)
+        if mrg is not main:
+            mrg.wait_event(att)
+        pipe.readout_merge(F("z", t), F("x", t), F("x", t), stream=mrg)
         ev = torch.cuda.Event(enable_timing=timers is not None)
-        ev.record(main)
-        rd_ev[t] = ev
+        ev.record(mrg)
+        rd_ev[t] = ev                        # frame t's keep-set and workspace are free
         if t + 1 < data.T and OVERLAP != "readout":
             issue_select(t + 1, after=ev)    # beside this frame's commit
-        pipe.commit(F("k", t), F("v", t), F("mask", t), 0)
         if timers is not None:
             e[1] = ev
             e[2].record(main)
-            timers.append((t, [sel_t[t][0], sel_t[t][1], e[0], e[1], e[2]]))
-    join = torch.cuda.Event()
-    join.record(side)
-    main.wait_event(join)
+        pipe.commit(F("k", t), F("v", t), F("mask", t), 0)
+        if timers is not None:
+            e[3].record(main)
+            timers.append((t, [sel_t[t][0], sel_t[t][1], e[0], e[1], e[2], e[3]]))
+    for st in (side, mrg):
+        if st is not main:
+            join = torch.cuda.Event()
+            join.record(st)
+            main.wait_event(join)
 
 
 def frame_work(w, counts, bank_lens, kw_lens):
@@ -340,6 +358,7 @@ def gpu_arm(args):
     def build(dense):
         data = DeviceSequence(w, dense, device)
         pipe = Pipeline(w, device=device, dense=dense)
+        torch.cuda.synchronize()        # inputs and bank set-up ran on the default stream
         return pipe, data
 
     results = {}
@@ -347,23 +366,24 @@ def gpu_arm(args):
         pipe, data = build(mode == "dense")
         stream = torch.cuda.Stream()
         side = torch.cuda.Stream()      # selection of frame t+1 runs beside frame t
+        merge = torch.cuda.Stream()     # split-KV merge of frame t beside its commit
         with torch.cuda.stream(stream):
             # warm-up (also sets kernel attributes before capture)
             for _ in range(max(args.warmup, 1)):
-                run_step(pipe, data, side=side)
+                run_step(pipe, data, side=side, merge=merge)
             torch.cuda.synchronize()
             work = work_model(pipe, data)
             torch.cuda.synchronize()
             # per-call timing pass (events on each call's launching stream)
             timers = []
-            run_step(pipe, data, timers, side=side)
+            run_step(pipe, data, timers, side=side, merge=merge)
             torch.cuda.synchronize()
             sel_ms = [t[1][0].elapsed_time(t[1][1]) for t in timers]
             rd_ms = [t[1][2].elapsed_time(t[1][3]) for t in timers]
-            cm_ms = [t[1][3].elapsed_time(t[1][4]) for t in timers]
+            cm_ms = [t[1][4].elapsed_time(t[1][5]) for t in timers]
             graph = torch.cuda.CUDAGraph()
             with torch.cuda.graph(graph, stream=stream):
-                run_step(pipe, data, side=side)
+                run_step(pipe, data, side=side, merge=merge)
             for _ in range(args.warmup):
                 graph.replay()
             torch.cuda.synchronize()
@@ -605,9 +625,12 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--overlap", default="readout", choices=["commit", "readout", "none"])
+    ap.add_argument("--merge-stream", default="on", choices=["on", "off"],
+                    help="run the readout's split-KV merge on its own stream beside the commit")
     args = ap.parse_args()
-    global OVERLAP
+    global OVERLAP, SPLIT_MERGE
     OVERLAP = args.overlap
+    SPLIT_MERGE = args.merge_stream == "on"
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
     if args.impl == "reference":

@@ -295,6 +295,34 @@ rs3_status rs3_memory_readout(const void *q, rs3_dtype dtype, int G, int mn, int
                               void *workspace, size_t workspace_bytes, int32_t *status,
                               rs3_stream_t stream);
 
+/*
+ * The same readout in two phases, with the arguments of rs3_memory_readout
+ * (the same values must be passed to both calls of one readout):
+ *   rs3_memory_readout_attend   the attention over the bank: writes the rows
+ *                               of unsplit work directly and leaves split-KV
+ *                               partial results in `workspace`;
+ *   rs3_memory_readout_merge    merges those partials and writes their rows.
+ * attend then merge on one stream is exactly rs3_memory_readout (same kernels,
+ * same results bit for bit).  The merge reads only the workspace, idx, count,
+ * unit_group, residual and out, never the bank, so once attend has completed
+ * a commit to the bank (Eq. 8, the write side of the same frame) may run on
+ * another stream concurrently with the merge.  Ordering is the caller's:
+ * merge after attend (e.g. through an event), the next attend or any other
+ * use of the same workspace after merge, and readers of `out` after merge.
+ */
+rs3_status rs3_memory_readout_attend(const void *q, rs3_dtype dtype, int G, int mn, int H, int d,
+                                     const int32_t *unit_group, const int32_t *idx,
+                                     const int32_t *count, int k_max, const rs3_bank *bank,
+                                     const float *rope, const void *residual, void *out, float scale,
+                                     void *workspace, size_t workspace_bytes, int32_t *status,
+                                     rs3_stream_t stream);
+rs3_status rs3_memory_readout_merge(const void *q, rs3_dtype dtype, int G, int mn, int H, int d,
+                                    const int32_t *unit_group, const int32_t *idx,
+                                    const int32_t *count, int k_max, const rs3_bank *bank,
+                                    const float *rope, const void *residual, void *out, float scale,
+                                    void *workspace, size_t workspace_bytes, int32_t *status,
+                                    rs3_stream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* Write side: keep-set (Sec. 3.2; Eq. 8)                                    */
 /* ------------------------------------------------------------------------ */

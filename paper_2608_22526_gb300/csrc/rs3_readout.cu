@@ -686,19 +686,21 @@ rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, in
     return RS3_OK;
 }
 
-rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_t max_items,
-                              int64_t max_combine, rs3_dtype dtype, cudaStream_t st)
+namespace {
+
+// pass-through of the unselected cells (out of place only), plan, attention
+rs3_status launch_attend(const ReadoutArgs &a, const ReadoutPath &p, rs3_dtype dtype, cudaStream_t st)
 {
     if (a.residual != a.out) {
         const int64_t nvec = (int64_t)a.U * a.mn * a.D * (dtype == RS3_BF16 ? 2 : 4) / 16;
         int64_t blocks = (nvec + 255) / 256;
         const int64_t cap = (int64_t)a.n_sm * 8;
         if (blocks > cap) blocks = cap;
-        launch_pdl(k_passthrough, dim3((unsigned)blocks), dim3(256), 0, st, static_cast<const uint4 *>(a.residual),
-                                                        static_cast<uint4 *>(a.out), nvec);
+        launch_pdl(k_passthrough, dim3((unsigned)blocks), dim3(256), 0, st,
+                   static_cast<const uint4 *>(a.residual), static_cast<uint4 *>(a.out), nvec);
         if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     }
-    // plan shared memory: unit slot bases and widths, per-CTA counts
+    // plan shared memory: unit slot bases and widths, slice bounds, per-CTA counts, unit tiles
     const size_t plan_smem = ((size_t)(2 * a.U + 1) + 2 * (size_t)(a.grid_ctas + 1)) * 8 + (size_t)a.U * 4;
     static size_t plan_attr = 0;
     if (plan_smem > 48 * 1024 && plan_smem > plan_attr) {
@@ -709,27 +711,27 @@ rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_
     }
     launch_pdl(k_plan, dim3(1), dim3(PLAN_THREADS), plan_smem, st, a);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
-    (void)max_items;
-    if (p.kind == 1) {
-        const rs3_status s = rs3_launch_tc_readout(a, st);
-        if (s != RS3_OK) return s;
-    } else {
-        const size_t smem = (size_t)2 * SIMT_BN * a.d * sizeof(float);
-        const int threads = 2 * a.d;
-        const int64_t blocks = a.grid_ctas;
-        static bool attr_done = false;
-        if (!attr_done) {
-            const int most = 2 * SIMT_BN * 256 * (int)sizeof(float);
-            cudaFuncSetAttribute(k_readout_simt<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
-            cudaFuncSetAttribute(k_readout_simt<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
-            attr_done = true;
-        }
-        if (dtype == RS3_BF16)
-            launch_pdl(k_readout_simt<uint16_t>, dim3((unsigned)blocks), dim3(threads), smem, st, a);
-        else
-            launch_pdl(k_readout_simt<float>, dim3((unsigned)blocks), dim3(threads), smem, st, a);
-        if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
+    if (p.kind == 1) return rs3_launch_tc_readout(a, st);
+    const size_t smem = (size_t)2 * SIMT_BN * a.d * sizeof(float);
+    const int threads = 2 * a.d;
+    const int64_t blocks = a.grid_ctas;
+    static bool attr_done = false;
+    if (!attr_done) {
+        const int most = 2 * SIMT_BN * 256 * (int)sizeof(float);
+        cudaFuncSetAttribute(k_readout_simt<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+        cudaFuncSetAttribute(k_readout_simt<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+        attr_done = true;
     }
+    if (dtype == RS3_BF16)
+        launch_pdl(k_readout_simt<uint16_t>, dim3((unsigned)blocks), dim3(threads), smem, st, a);
+    else
+        launch_pdl(k_readout_simt<float>, dim3((unsigned)blocks), dim3(threads), smem, st, a);
+    return cudaGetLastError() == cudaSuccess ? RS3_OK : RS3_ECUDA;
+}
+
+// merge of the split-KV partials and their scatter
+rs3_status launch_merge(const ReadoutArgs &a, int64_t max_combine, rs3_dtype dtype, cudaStream_t st)
+{
     // one warp per (partial row, 64-column chunk; 32 for d < 64)
     const int ce = a.d >= 64 ? 2 : 1;
     const int64_t chunks = (a.d + 32 * ce - 1) / (32 * ce);
@@ -744,16 +746,29 @@ rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_
         if (ce == 2) launch_pdl(k_combine<float, 2>, dim3((unsigned)cblocks), dim3(256), 0, st, a);
         else launch_pdl(k_combine<float, 1>, dim3((unsigned)cblocks), dim3(256), 0, st, a);
     }
-    if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
+    return cudaGetLastError() == cudaSuccess ? RS3_OK : RS3_ECUDA;
+}
+
+}  // namespace
+
+rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_t max_items,
+                              int64_t max_combine, rs3_dtype dtype, cudaStream_t st, int phases)
+{
+    (void)max_items;
+    if (phases & RS3_PHASE_ATTEND) {
+        const rs3_status s = launch_attend(a, p, dtype, st);
+        if (s != RS3_OK) return s;
+    }
+    if (phases & RS3_PHASE_MERGE) return launch_merge(a, max_combine, dtype, st);
     return RS3_OK;
 }
 
-extern "C" rs3_status rs3_memory_readout(const void *q, rs3_dtype dtype, int G, int mn, int H,
-                                         int d, const int32_t *unit_group, const int32_t *idx,
-                                         const int32_t *count, int k_max, const rs3_bank *bank,
-                                         const float *rope, const void *residual, void *out,
-                                         float scale, void *workspace, size_t workspace_bytes,
-                                         int32_t *status, rs3_stream_t stream)
+namespace {
+
+rs3_status readout_call(const void *q, rs3_dtype dtype, int G, int mn, int H, int d, const int32_t *unit_group,
+                        const int32_t *idx, const int32_t *count, int k_max, const rs3_bank *bank,
+                        const float *rope, const void *residual, void *out, float scale, void *workspace,
+                        size_t workspace_bytes, int32_t *status, rs3_stream_t stream, int phases)
 {
     ReadoutArgs a;
     ReadoutPath p;
@@ -762,5 +777,40 @@ extern "C" rs3_status rs3_memory_readout(const void *q, rs3_dtype dtype, int G, 
                                              bank, rope, residual, out, scale, workspace,
                                              workspace_bytes, status, &a, &p, &gi, &gc);
     if (s != RS3_OK) return s;
-    return rs3_readout_launch(a, p, gi, gc, dtype, reinterpret_cast<cudaStream_t>(stream));
+    return rs3_readout_launch(a, p, gi, gc, dtype, reinterpret_cast<cudaStream_t>(stream), phases);
+}
+
+}  // namespace
+
+extern "C" rs3_status rs3_memory_readout(const void *q, rs3_dtype dtype, int G, int mn, int H,
+                                         int d, const int32_t *unit_group, const int32_t *idx,
+                                         const int32_t *count, int k_max, const rs3_bank *bank,
+                                         const float *rope, const void *residual, void *out,
+                                         float scale, void *workspace, size_t workspace_bytes,
+                                         int32_t *status, rs3_stream_t stream)
+{
+    return readout_call(q, dtype, G, mn, H, d, unit_group, idx, count, k_max, bank, rope, residual, out, scale,
+                        workspace, workspace_bytes, status, stream, RS3_PHASE_ATTEND | RS3_PHASE_MERGE);
+}
+
+extern "C" rs3_status rs3_memory_readout_attend(const void *q, rs3_dtype dtype, int G, int mn, int H,
+                                                int d, const int32_t *unit_group, const int32_t *idx,
+                                                const int32_t *count, int k_max, const rs3_bank *bank,
+                                                const float *rope, const void *residual, void *out,
+                                                float scale, void *workspace, size_t workspace_bytes,
+                                                int32_t *status, rs3_stream_t stream)
+{
+    return readout_call(q, dtype, G, mn, H, d, unit_group, idx, count, k_max, bank, rope, residual, out, scale,
+                        workspace, workspace_bytes, status, stream, RS3_PHASE_ATTEND);
+}
+
+extern "C" rs3_status rs3_memory_readout_merge(const void *q, rs3_dtype dtype, int G, int mn, int H,
+                                               int d, const int32_t *unit_group, const int32_t *idx,
+                                               const int32_t *count, int k_max, const rs3_bank *bank,
+                                               const float *rope, const void *residual, void *out,
+                                               float scale, void *workspace, size_t workspace_bytes,
+                                               int32_t *status, rs3_stream_t stream)
+{
+    return readout_call(q, dtype, G, mn, H, d, unit_group, idx, count, k_max, bank, rope, residual, out, scale,
+                        workspace, workspace_bytes, status, stream, RS3_PHASE_MERGE);
 }

@@ -62,6 +62,24 @@ class Pipeline:
                                self.count, self.k_max, self.bank, rope, residual, out, scale,
                                self.ws_readout, self.status, self.stream)
 
+    def readout_attend(self, q: torch.Tensor, residual: Optional[torch.Tensor], out: torch.Tensor,
+                       rope: Optional[torch.Tensor] = None, scale: float = 0.0, stream=None):
+        """First phase of readout(): the attention over the bank."""
+        w = self.w
+        rs3.rs3_memory_readout_attend(q, w.dtype, w.G, w.mn, w.H, w.d, self.unit_group, self.idx,
+                                      self.count, self.k_max, self.bank, rope, residual, out, scale,
+                                      self.ws_readout, self.status,
+                                      stream if stream is not None else self.stream)
+
+    def readout_merge(self, q: torch.Tensor, residual: Optional[torch.Tensor], out: torch.Tensor,
+                      rope: Optional[torch.Tensor] = None, scale: float = 0.0, stream=None):
+        """Second phase of readout(): the split-KV merge; reads no bank."""
+        w = self.w
+        rs3.rs3_memory_readout_merge(q, w.dtype, w.G, w.mn, w.H, w.d, self.unit_group, self.idx,
+                                     self.count, self.k_max, self.bank, rope, residual, out, scale,
+                                     self.ws_readout, self.status,
+                                     stream if stream is not None else self.stream)
+
     def commit(self, k_new: torch.Tensor, v_new: torch.Tensor, mask: Optional[torch.Tensor],
                is_cond: int):
         rs3.rs3_bank_commit(self.bank, k_new, v_new, None if self.dense else mask, is_cond,

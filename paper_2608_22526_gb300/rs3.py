@@ -68,6 +68,10 @@ SIGNATURES = {
     "rs3_readout_workspace_bytes": (_SZ, [_I, _I, _I, _I, _I]),
     "rs3_memory_readout": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P, _P, _P, _P,
                                 ctypes.c_float, _P, _SZ, _P, _P]),
+    "rs3_memory_readout_attend": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P, _P, _P, _P,
+                                ctypes.c_float, _P, _SZ, _P, _P]),
+    "rs3_memory_readout_merge": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P, _P, _P, _P,
+                                ctypes.c_float, _P, _SZ, _P, _P]),
     "rs3_write_keepset": (_I, [_P, _P, _I, _I, _I, _P, _P, _P, _P]),
 }
 
@@ -165,6 +169,28 @@ def rs3_memory_readout(q, dtype: str, G: int, mn: int, H: int, d: int, unit_grou
                                 workspace.numel() * workspace.element_size(), _ptr(status),
                                 _stream(stream))
     _check(rc, "rs3_memory_readout")
+
+
+def _readout_phase(fn, name, q, dtype, G, mn, H, d, unit_group, idx, count, k_max, bank, rope, residual,
+                   out, scale, workspace, status, stream):
+    rc = fn(_ptr(q), DTYPES[dtype], G, mn, H, d, _ptr(unit_group), _ptr(idx), _ptr(count), k_max,
+            ctypes.byref(bank.desc), _ptr(rope), _ptr(residual), _ptr(out), float(scale), _ptr(workspace),
+            workspace.numel() * workspace.element_size(), _ptr(status), _stream(stream))
+    _check(rc, name)
+
+
+def rs3_memory_readout_attend(q, dtype: str, G: int, mn: int, H: int, d: int, unit_group, idx, count,
+                              k_max: int, bank: "Bank", rope, residual, out, scale: float, workspace,
+                              status, stream=None):
+    _readout_phase(lib.rs3_memory_readout_attend, "rs3_memory_readout_attend", q, dtype, G, mn, H, d,
+                   unit_group, idx, count, k_max, bank, rope, residual, out, scale, workspace, status, stream)
+
+
+def rs3_memory_readout_merge(q, dtype: str, G: int, mn: int, H: int, d: int, unit_group, idx, count,
+                             k_max: int, bank: "Bank", rope, residual, out, scale: float, workspace,
+                             status, stream=None):
+    _readout_phase(lib.rs3_memory_readout_merge, "rs3_memory_readout_merge", q, dtype, G, mn, H, d,
+                   unit_group, idx, count, k_max, bank, rope, residual, out, scale, workspace, status, stream)
 
 
 def rs3_write_keepset(seed_masks, unit_group, U: int, m: int, n: int, params: Params, kw_out,
