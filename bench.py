@@ -225,8 +225,9 @@ def run_step(pipe, data, timers=None, side=None, merge=None):
     from paper_2608_22526_gb300 import rs3
     main = torch.cuda.current_stream()
     side = side if (side is not None and OVERLAP != "none") else main
-    # the per-call timing pass (timers) keeps each frame's calls back to back
-    # on one stream, so that their event times are the calls' own durations
+    # the per-call timing pass (timers) issues each frame's calls back to back
+    # on one stream, the readout as one call, so that their event times are
+    # the calls' own durations
     mrg = merge if (merge is not None and SPLIT_MERGE and timers is None) else main
     rs3.rs3_bank_reset(pipe.bank, -1)
     pipe.track.zero_()
@@ -274,12 +275,14 @@ def run_step(pipe, data, timers=None, side=None, merge=None):
         if timers is not None:
             e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
             e[0].record(main)
-        pipe.readout_attend(F("z", t), F("x", t), F("x", t))
-        att = torch.cuda.Event(enable_timing=timers is not None)
-        att.record(main)
-        if mrg is not main:
+        if mrg is main:
+            pipe.readout(F("z", t), F("x", t), F("x", t))        # both phases, one call
+        else:
+            pipe.readout_attend(F("z", t), F("x", t), F("x", t))
+            att = torch.cuda.Event()
+            att.record(main)
             mrg.wait_event(att)
-        pipe.readout_merge(F("z", t), F("x", t), F("x", t), stream=mrg)
+            pipe.readout_merge(F("z", t), F("x", t), F("x", t), stream=mrg)
         ev = torch.cuda.Event(enable_timing=timers is not None)
         ev.record(mrg)
         rd_ev[t] = ev                        # frame t's keep-set and workspace are free
