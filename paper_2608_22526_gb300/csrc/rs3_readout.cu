@@ -2,7 +2,7 @@
 // scatter, Eq. 7 RoPE by the gathered index), host entry and the shared
 // pieces of both kernel paths.
 //
-// Launch sequence (one stream, no host synchronisation):
+// Launch sequence (no host synchronisation).  Attend phase:
 //   k_passthrough  out-of-place only: out = residual (or zeros) on every cell
 //   k_plan         one CTA: per unit, the bank's row ranges (pinned, ring
 //                  pieces, pointers) and a balanced work list of
@@ -13,7 +13,10 @@
 //                  log2 domain, fp32 accumulation; an unsplit item writes
 //                  out = residual + A directly at the kept cells, a split item
 //                  writes (O, m, l) partials
+// Merge phase (reads no bank, so it may run beside a commit):
 //   k_combine      log-sum-exp merge of the partials and the scatter
+// rs3_memory_readout issues both phases on one stream;
+// rs3_memory_readout_attend / _merge issue one each.
 #include "rs3_internal.cuh"
 
 #include <cmath>
