@@ -376,7 +376,7 @@ void or_round_bf16_array(const double *x, long n, uint16_t *out)
 
 /* K_w per unit.  S = the unit's seed mask, or in union mode the union of the
  * seeds of its group.  If fall_through is set and |S|/mn > hi or < lo, K_w is
- * the full grid (Sec. 3.2, "falls through to the original write path");
+ * the full grid (Sec. 3.2: such frames are written unpruned);
  * otherwise K_w = dilate_{D_w}(S) (the union of per-object dilations equals
  * the dilation of the union). */
 void or_write_keepset(const uint8_t *seeds, const int32_t *unit_group, int U, int m, int n,
