@@ -1,0 +1,57 @@
+"""Host-side pieces of bench.py that need no GPU: the algorithmic work a
+frame is credited with, the key that ties a stored ncu traffic figure to the
+readout sources, and the config string of every workload."""
+import os
+import shutil
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+import bench  # noqa: E402
+from paper_2608_22526_gb300 import synth  # noqa: E402
+
+
+def test_frame_work_closed_form():
+    w = synth.WORKLOADS["sam2_8obj"]
+    counts = [1228, 600, 0, 5, 1228, 1000, 1, 300]
+    banks = [5000, 4000, 7000, 0, 100, 6000, 28672, 16]
+    kw = [800, 0, 1600, 4096, 10, 20, 30, 40]
+    flops, cbytes = bench.frame_work(w, counts, banks, kw)
+    # Eq. 6 per unit: q~ K^T and P V, each 2 |K_r| N d flops per head
+    assert flops == sum(4.0 * c * n * w.H * w.d for c, n in zip(counts, banks))
+    # commit: every unit's mask, K and V rows read and written (bf16)
+    assert cbytes == w.U * w.mn + sum(4 * L * w.D * 2 for L in kw)
+
+
+def test_traffic_key_ignores_comments_not_code(tmp_path, monkeypatch):
+    src = os.path.join(ROOT, "paper_2608_22526_gb300", "csrc")
+    dst = tmp_path / "paper_2608_22526_gb300" / "csrc"
+    dst.mkdir(parents=True)
+    for f in ("rs3_readout.cu", "rs3_readout_tc.cu", "rs3_readout_common.cuh", "rs3_tc_ptx.cuh"):
+        shutil.copy(os.path.join(src, f), dst / f)
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    h0 = bench.readout_source_hash()
+    p = dst / "rs3_readout.cu"
+    text = p.read_text()
+    p.write_text("// a new comment line\n/* and a block\n   comment */\n" + text.replace("\n", "\n\n", 3))
+    assert bench.readout_source_hash() == h0
+    p.write_text(text.replace("a->plan_ov = p.kind == 1 ? 12 : 1;", "a->plan_ov = p.kind == 1 ? 13 : 1;"))
+    assert bench.readout_source_hash() != h0
+
+
+def test_traffic_record_matches_the_committed_sources():
+    """profiles/traffic.json was taken on the readout kernel as committed."""
+    rec = bench._traffic_record(synth.WORKLOADS["sam2_1obj"])
+    assert rec is not None and rec > 0
+
+
+@pytest.mark.parametrize("name", sorted(synth.WORKLOADS))
+def test_workload_config_names_the_workload(name):
+    w = synth.WORKLOADS[name]
+    cfg = bench.workload_config(w, 1)
+    assert cfg["workload"].startswith(name + ":")
+    assert f"{w.m}x{w.n}" in cfg["workload"] and f"{w.frames} frames" in cfg["workload"]
+    assert cfg["parallelism"] == "replicas x1"
