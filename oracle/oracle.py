@@ -13,6 +13,9 @@ memory bank.  Each function cites the part of the paper it follows:
   scatter_output() Sec. 3.1: Eq. 6 scatter S_K back onto the m x n grid
   OracleBank       Sec. 3.2: Eq. 8 write-pruned commit, Algorithm 1 sparse write
   write_keepset()  Sec. 3.2: Eq. 8 with the 5% / 95% fall-through
+  close_argmax()   Sec. 3.3: 9 x 9 closure per object, then the palette argmax
+  downsample(), seed_track()
+                   Sec. 3.1: down_s of pixel masks, the seed box of Eq. 1
 """
 from __future__ import annotations
 
@@ -68,6 +71,12 @@ def _lib():
             lib.or_commit_unit.argtypes = [P, P, i64, P, P, P, i64, i32, i32, i64, i64, i32,
                                            P, P, P]
             lib.or_commit_unit.restype = i32
+            lib.or_erode.argtypes = [P, i32, i32, i32, P]
+            lib.or_close.argtypes = [P, i32, i32, i32, P]
+            lib.or_close_argmax.argtypes = [P, i32, i32, i32, i32, P, P]
+            lib.or_downsample.argtypes = [P, i32, i32, i32, P]
+            lib.or_seed_track.argtypes = [P, i32, i32, i32, P]
+            lib.or_seed_track.restype = i32
             _handle = lib
     return _handle
 
@@ -330,3 +339,51 @@ class OracleBank:
         n, o = int(self.state[u, 3]), int(self.state[u, 4])
         return [(int(self.foff[u, (o + i) % self.max_frames]),
                  int(self.flen[u, (o + i) % self.max_frames])) for i in range(n)]
+
+
+# ---------------------------------------------------------------------------
+# decoder side (Sec. 3.3) and the pixel-space front end (Sec. 3.1)
+# ---------------------------------------------------------------------------
+
+def erode(M: np.ndarray, h: int, w: int, r: int) -> np.ndarray:
+    """Square erosion by r with the window clipped to the image."""
+    out = np.empty(h * w, dtype=np.uint8)
+    _lib().or_erode(_p(_c(M, np.uint8)), h, w, int(r), _p(out))
+    return out.reshape(h, w)
+
+
+def close(M: np.ndarray, h: int, w: int, r: int) -> np.ndarray:
+    """close_r(M) = erode_r(dilate_r(M)) (Sec. 3.3: r = 4, the 9 x 9 square)."""
+    out = np.empty(h * w, dtype=np.uint8)
+    _lib().or_close(_p(_c(M, np.uint8)), h, w, int(r), _p(out))
+    return out.reshape(h, w)
+
+
+def close_argmax(logits: np.ndarray, r: int):
+    """One group: logits [nobj, h, w] fp32 -> (closed [nobj, h, w] uint8,
+    palette [h, w] uint8 with 0 = background and 1 + o = object o)."""
+    L = _c(logits, np.float32)
+    nobj, h, w = L.shape
+    closed = np.empty((nobj, h, w), dtype=np.uint8)
+    palette = np.empty((h, w), dtype=np.uint8)
+    _lib().or_close_argmax(_p(L), nobj, h, w, int(r), _p(closed), _p(palette))
+    return closed, palette
+
+
+def downsample(M: np.ndarray, s: int) -> np.ndarray:
+    """down_s: grid cell (i, j) takes pixel (i*s, j*s); [h, w] -> [h/s, w/s]."""
+    M = _c(M, np.uint8)
+    h, w = M.shape
+    out = np.empty((h // s, w // s), dtype=np.uint8)
+    _lib().or_downsample(_p(M), h, w, int(s), _p(out))
+    return out
+
+
+def seed_track(M: np.ndarray, s: int) -> np.ndarray:
+    """The seed box of Eq. 1 on the grid: int32 [6] = (y0, x0, y1, x1, valid,
+    streak) from the tight pixel box of M, corners divided by s (floor)."""
+    M = _c(M, np.uint8)
+    h, w = M.shape
+    t = np.zeros(6, dtype=np.int32)
+    _lib().or_seed_track(_p(M), h, w, int(s), _p(t))
+    return t

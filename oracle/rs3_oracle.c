@@ -14,6 +14,8 @@
  *                           scatter) and Eq. 7 (RoPE by the gathered index)
  *   commit                  Sec. 3.2, Eq. 8 and Algorithm 1 (sparse write)
  *   write keep-set          Sec. 3.2, Eq. 8 and the 5%/95% fall-through
+ *   closure + palette       Sec. 3.3 (9 x 9 closure per object, then argmax)
+ *   down_s + seed box       Sec. 3.1 (pixel masks and boxes onto the grid)
  *
  * Readings where the paper is silent or ambiguous (documented in the design doc):
  *   - dilate_r is a Chebyshev (square) dilation by r cells;
@@ -22,7 +24,14 @@
  *   - energies are ranked in a canonical fp32 order (see or_energy_canonical);
  *     ties go to the lower grid index; the keep-set is emitted in ascending
  *     grid order; k = floor(rho * mn) (Table 4 lists 819/1228/2048/2867/4096);
- *   - the score scale is 1/sqrt(d) per head; an empty bank reads out zeros.
+ *   - the score scale is 1/sqrt(d) per head; an empty bank reads out zeros;
+ *   - a decoder mask is logit > 0; the closure treats the object as a set of
+ *     the unbounded plane with nothing set outside the image (so it neither
+ *     grows an object out to the border nor erodes one that touches it); the
+ *     palette gives each pixel to the object with the largest logit among
+ *     those whose closed mask holds it, the lower object on equal logits;
+ *   - down_s samples pixel (i*s, j*s) for grid cell (i, j); a pixel box maps
+ *     onto the grid by dividing each corner by s, rounding down.
  */
 #include <math.h>
 #include <pthread.h>
@@ -461,4 +470,104 @@ int or_commit_unit(uint8_t *kst, uint8_t *vst, long row_bytes, const uint8_t *kn
     state[3] = n_frames + 1;
     state[4] = oldest;
     return 0;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Decoder side (Sec. 3.3): per-object closure, then the palette argmax      */
+/* ------------------------------------------------------------------------- */
+
+/* out(y,x) = 1 iff every pixel (y',x') of the array with |y-y'| <= r and
+ * |x-x'| <= r is set (the window clipped to the array). */
+void or_erode(const uint8_t *M, int h, int w, int r, uint8_t *out)
+{
+    for (int y = 0; y < h; ++y)
+        for (int x = 0; x < w; ++x) {
+            int all = 1;
+            for (int yy = y - r; yy <= y + r && all; ++yy) {
+                if (yy < 0 || yy >= h) continue;
+                for (int xx = x - r; xx <= x + r; ++xx) {
+                    if (xx < 0 || xx >= w) continue;
+                    if (!M[(long)yy * w + xx]) { all = 0; break; }
+                }
+            }
+            out[(long)y * w + x] = (uint8_t)all;
+        }
+}
+
+/* Closure with the (2r+1) x (2r+1) square: dilation, then erosion (Sec. 3.3
+ * uses r = 4, a 9 x 9 element).  The object is a set of pixels of the
+ * unbounded plane with nothing set outside the image; both operations are
+ * taken in the plane and the result is cut back to the image.  Written out:
+ * the image is embedded in a zero frame 2r pixels wide, where no clipped
+ * window of the two passes reaches the frame's edge for the pixels kept. */
+void or_close(const uint8_t *M, int h, int w, int r, uint8_t *out)
+{
+    int H = h + 4 * r, W = w + 4 * r;
+    uint8_t *pad = (uint8_t *)calloc((size_t)H * W, 1);
+    uint8_t *dil = (uint8_t *)malloc((size_t)H * W);
+    uint8_t *ero = (uint8_t *)malloc((size_t)H * W);
+    for (int y = 0; y < h; ++y)
+        for (int x = 0; x < w; ++x) pad[(long)(y + 2 * r) * W + (x + 2 * r)] = M[(long)y * w + x];
+    or_dilate(pad, H, W, r, dil);
+    or_erode(dil, H, W, r, ero);
+    for (int y = 0; y < h; ++y)
+        for (int x = 0; x < w; ++x) out[(long)y * w + x] = ero[(long)(y + 2 * r) * W + (x + 2 * r)];
+    free(pad);
+    free(dil);
+    free(ero);
+}
+
+/* One group of nobj objects at the decoder's resolution h x w.
+ *   logits  [nobj][h][w] fp32 decoder mask logits; object o's binary mask is
+ *           logit > 0
+ *   closed  [nobj][h][w] out: close_r of each object's mask
+ *   palette [h][w] out: 0 where no closed mask holds the pixel, otherwise
+ *           1 + o for the object o with the largest logit among the objects
+ *           whose closed mask holds it (the lower o on equal logits).
+ * The closure comes first and the argmax second, the order of Sec. 3.3. */
+void or_close_argmax(const float *logits, int nobj, int h, int w, int r, uint8_t *closed,
+                     uint8_t *palette)
+{
+    long hw = (long)h * w;
+    uint8_t *bin = (uint8_t *)malloc((size_t)hw);
+    for (int o = 0; o < nobj; ++o) {
+        for (long i = 0; i < hw; ++i) bin[i] = logits[(long)o * hw + i] > 0.0f;
+        or_close(bin, h, w, r, closed + (long)o * hw);
+    }
+    for (long i = 0; i < hw; ++i) {
+        int best = -1;
+        for (int o = 0; o < nobj; ++o) {
+            if (!closed[(long)o * hw + i]) continue;
+            if (best < 0 || logits[(long)o * hw + i] > logits[(long)best * hw + i]) best = o;
+        }
+        palette[i] = (uint8_t)(best + 1);
+    }
+    free(bin);
+}
+
+/* ------------------------------------------------------------------------- */
+/* Pixel space to token grid (Sec. 3.1: down_s and the seed box of Eq. 1)    */
+/* ------------------------------------------------------------------------- */
+
+/* Nearest-neighbour down_s: grid cell (i, j) of the (h/s) x (w/s) grid takes
+ * pixel (i*s, j*s). */
+void or_downsample(const uint8_t *M, int h, int w, int s, uint8_t *out)
+{
+    int m = h / s, n = w / s;
+    for (int i = 0; i < m; ++i)
+        for (int j = 0; j < n; ++j) out[(long)i * n + j] = M[(long)i * s * w + (long)j * s] != 0;
+}
+
+/* Seed of one object: the tight pixel box of M (inclusive), each corner
+ * coordinate divided by s with the quotient rounded down.  track = {y0, x0,
+ * y1, x1, valid, streak}: valid 1 and streak 0 when M has a set pixel; an
+ * empty M gives {0, 0, 0, 0, 0, 0}.  Returns valid. */
+int or_seed_track(const uint8_t *M, int h, int w, int s, int32_t *track)
+{
+    int32_t box[4];
+    for (int k = 0; k < 6; ++k) track[k] = 0;
+    if (!or_bbox(M, h, w, box)) return 0;
+    for (int k = 0; k < 4; ++k) track[k] = box[k] / s;
+    track[4] = 1;
+    return 1;
 }
