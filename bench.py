@@ -31,6 +31,9 @@ sys.path.insert(0, ROOT)
 METRIC = "pruned readout frames/s & TFLOP/s vs dense (1 GB300); bank-commit HBM GB/s"
 WORKLOAD = "sam2_1obj"
 KERNELS_PER_READOUT_FRAME = 7     # prior, energy, select, plan, readout, combine, commit
+DECODER_STRIDE = 4                # decoder masks at 4x the token grid (SAM2: 256^2 masks, 64^2 tokens)
+CLOSE_RADIUS = 4                  # the 9 x 9 closure of Sec. 3.3
+L2_BYTES = 129 * 2 ** 20
 
 
 def _peaks():
@@ -542,12 +545,70 @@ def gpu_arm(args):
         line["e2e"] = {"value": round(e2e_val, 2), "unit": "frames/s",
                        "h2d_bytes_per_step": int(P["e2e_bytes"][0]),
                        "d2h_bytes_per_step": int(P["e2e_bytes"][1])}
+    if not args.no_decoder:
+        line["close_argmax"] = measure_close_argmax(w, device, hbm)
     if not args.no_cpu_baseline and world == 1:
         line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_seconds)
     print(json.dumps(line), flush=True)
     if world > 1:
         dist.barrier()
         dist.destroy_process_group()
+
+
+def close_argmax_work(w):
+    """Algorithmic bytes of one rs3_close_argmax launch over the workload's
+    streams at the decoder's resolution: every object's fp32 logits read, the
+    palette and the grid masks written."""
+    h, wd = DECODER_STRIDE * w.m, DECODER_STRIDE * w.n
+    return w.U * h * wd * 4 + w.G * h * wd + w.U * w.mn
+
+
+def measure_close_argmax(w, device, hbm, launches=200):
+    """The decoder-side kernel (Sec. 3.3) on its own: per-object closure,
+    palette argmax and down_s of the closed masks, timed with CUDA events on
+    its stream over `launches` back-to-back launches whose logits rotate
+    through distinct buffers totalling more than twice the L2."""
+    import torch
+    from paper_2608_22526_gb300 import rs3, synth
+    h, wd = DECODER_STRIDE * w.m, DECODER_STRIDE * w.n
+    if wd % 32 != 0:
+        return None
+    frame_bytes = w.U * h * wd * 4
+    nbuf = int(math.ceil(2 * L2_BYTES / frame_bytes)) + 1
+    logits = torch.from_numpy(synth.decoder_logits(np.random.default_rng(w.seed + 101), w.U, h, wd))
+    bufs = logits.to(device).unsqueeze(0).repeat(nbuf, 1, 1, 1).contiguous()
+    gs = torch.arange(0, w.U + 1, w.units_per_group, dtype=torch.int32, device=device)
+    pal = torch.empty((w.G, h, wd), dtype=torch.uint8, device=device)
+    grid = torch.empty((w.U, w.m, w.n), dtype=torch.uint8, device=device)
+    status = torch.zeros(1, dtype=torch.int32, device=device)
+    stream = torch.cuda.Stream(device)
+    torch.cuda.synchronize()
+
+    def launch(i):
+        rs3.rs3_close_argmax(bufs[i % nbuf], gs, w.G, w.U, h, wd, CLOSE_RADIUS, DECODER_STRIDE, pal,
+                             None, grid, status, stream=stream)
+
+    with torch.cuda.stream(stream):
+        for i in range(5):
+            launch(i)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(launches):
+            launch(5 + i)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0, "device status word set"
+    us = e0.elapsed_time(e1) * 1e3 / launches
+    nbytes = close_argmax_work(w)
+    gbs = nbytes / (us * 1e-6) / 1e9
+    del bufs
+    return {"kernel": "rs3_close_argmax (9x9 closure per object + palette argmax + down_s)",
+            "shape": f"{w.G} stream(s) x {w.units_per_group} object(s), {h}x{wd} fp32 logits, "
+                     f"{w.m}x{w.n} grid",
+            "us_per_launch": round(us, 3), "bytes_per_launch": int(nbytes),
+            "bound": "hbm", "achieved_gbs": round(gbs, 1), "peak_gbs": hbm, "frac": round(gbs / hbm, 4),
+            "inputs": f"{nbuf} distinct logit buffers in rotation (> 2x L2)"}
 
 
 def workload_config(w, world):
@@ -679,6 +740,7 @@ def main():
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-decoder", action="store_true", help="skip the decoder-side kernel measurement")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--overlap", default="readout", choices=["commit", "readout", "none"])

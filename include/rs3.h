@@ -14,6 +14,11 @@
  *                          rs3_bank_commit     -- append the kept tokens to a
  *                                                ragged per-unit bank
  *                                                (Algorithm 1, sparse write)
+ *   decoder side (Sec. 3.3) rs3_close_argmax   -- per-object 9 x 9 closure,
+ *                                                palette argmax, down_s of the
+ *                                                closed masks onto the grid
+ *   front end (Sec. 3.1)   rs3_seed_from_masks -- seed box of Eq. 1 from
+ *                                                pixel masks, down_s
  *
  * Vocabulary.  A *unit* is one (stream, object) pair: it owns one keep-set,
  * one memory bank and one output grid.  A *group* is the set of units that
@@ -21,7 +26,8 @@
  * m x n cells (mn = m*n), row-major, cell i = y*n + x.  D = H*d is the width
  * of a query / key / value row (H heads of dimension d; head h owns columns
  * [h*d, (h+1)*d)).  Masks are given at grid resolution (the down_s of
- * Eq. 1/2/8 already applied).
+ * Eq. 1/2/8 already applied), except where rs3_close_argmax and
+ * rs3_seed_from_masks take pixel-resolution input and apply it.
  *
  * Conventions for every call.
  *   - Device pointers are owned by the caller; the library never allocates,
@@ -339,6 +345,59 @@ rs3_status rs3_memory_readout_merge(const void *q, rs3_dtype dtype, int G, int m
 rs3_status rs3_write_keepset(const uint8_t *seed_masks, const int32_t *unit_group, int U, int m,
                              int n, const rs3_params *p, uint8_t *kw_out, int32_t *status,
                              rs3_stream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* Decoder side (Sec. 3.3) and the pixel-space front end (Sec. 3.1)          */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Per-frame post-processing of the mask decoder's output (Sec. 3.3,
+ * Algorithm 1 after the decoder): each object's binary mask (logit > 0) is
+ * closed with the (2*radius+1)^2 square -- a dilation, then an erosion; the
+ * paper uses radius 4, the 9 x 9 element -- and then every pixel goes to the
+ * object with the largest logit among the objects of its stream whose closed
+ * mask holds it (the palette mask; 0 = background; equal logits go to the
+ * object listed first).  The closure treats an object as a set of the
+ * unbounded plane with nothing set outside the image, so it is extensive and
+ * idempotent, fills holes and bridges gaps of at most 2*radius pixels, and
+ * neither grows an object out to the image border nor erodes one touching it.
+ *   logits      device fp32 [U][h][w], decoder mask logits at the decoder's
+ *               resolution (finite values)
+ *   group_start device int32 [G+1]: the objects of stream g are the units
+ *               [group_start[g], group_start[g+1]), at most 255 of them; a
+ *               stream whose range is not inside [0, U] or holds more than 255
+ *               objects latches RS3_EINVAL into *status and is skipped
+ *   palette     device uint8 [G][h][w] or NULL: 0, or 1 + the object's index
+ *               within its stream
+ *   closed      device uint8 [U][h][w] or NULL: each object's closed mask (0/1),
+ *               the per-object masks M_t|o that Algorithm 1's tracker reads
+ *   grid_masks  device uint8 [U][h/s][w/s] or NULL: down_s of each closed mask
+ *               (cell (i, j) takes pixel (i*s, j*s), Sec. 3.1), the previous-
+ *               frame masks that rs3_select_queries consumes next frame
+ *   status      device int32 word (see conventions)
+ * Limits: w a multiple of 32, 0 <= radius <= 8, G <= 65535; h and w multiples
+ * of s when grid_masks is given.
+ */
+rs3_status rs3_close_argmax(const float *logits, const int32_t *group_start, int G, int U, int h,
+                            int w, int radius, int s, uint8_t *palette, uint8_t *closed,
+                            uint8_t *grid_masks, int32_t *status, rs3_stream_t stream);
+
+/*
+ * Seed of every object from its pixel-resolution mask (Sec. 3.1, Eq. 1): the
+ * tight pixel box of the set pixels, each corner divided by the encoder
+ * stride s and rounded down, becomes the unit's tracker state ({y0, x0, y1,
+ * x1} on the grid, valid 1, streak 0; an empty mask gives all zeros), so the
+ * first rs3_select_queries call with an empty previous mask and bbox_mode, or
+ * with box_masks as the previous mask, dilates down_s of the seed box.
+ *   masks      device uint8 [U][h][w] (nonzero = set), 16-byte aligned
+ *   track      device rs3_track [U], written
+ *   grid_masks device uint8 [U][h/s][w/s] or NULL: down_s of the mask (cell
+ *              (i, j) takes pixel (i*s, j*s))
+ *   box_masks  device uint8 [U][h/s][w/s] or NULL: the projected box, filled
+ * Limits: w a multiple of 16; h and w multiples of s; U <= 65535.
+ */
+rs3_status rs3_seed_from_masks(const uint8_t *masks, int U, int h, int w, int s, rs3_track *track,
+                               uint8_t *grid_masks, uint8_t *box_masks, rs3_stream_t stream);
 
 #ifdef __cplusplus
 }

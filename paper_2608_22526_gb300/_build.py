@@ -18,7 +18,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "librs3.so")
 
 SOURCES = ["rs3_api.cu", "rs3_select.cu", "rs3_bank.cu", "rs3_readout.cu", "rs3_readout_tc.cu",
-           "rs3_noalloc.cu"]
+           "rs3_noalloc.cu", "rs3_masks.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
               "-I" + os.path.join(ROOT, "include")]

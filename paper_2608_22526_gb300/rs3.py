@@ -73,6 +73,8 @@ SIGNATURES = {
     "rs3_memory_readout_merge": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P, _P, _P, _P,
                                 ctypes.c_float, _P, _SZ, _P, _P]),
     "rs3_write_keepset": (_I, [_P, _P, _I, _I, _I, _P, _P, _P, _P]),
+    "rs3_close_argmax": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
+    "rs3_seed_from_masks": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P]),
 }
 
 
@@ -270,3 +272,21 @@ def rs3_bank_read_meta(bank: Bank, stream=None):
                                 fr.ctypes.data_as(ctypes.c_void_p), _stream(stream))
     _check(rc, "rs3_bank_read_meta")
     return out, fr
+
+
+# ---------------------------------------------------------------------------
+# decoder side and pixel-space front end
+# ---------------------------------------------------------------------------
+
+def rs3_close_argmax(logits, group_start, G: int, U: int, h: int, w: int, radius: int, s: int,
+                     palette, closed, grid_masks, status, stream=None):
+    rc = lib.rs3_close_argmax(_ptr(logits), _ptr(group_start), G, U, h, w, radius, s, _ptr(palette),
+                              _ptr(closed), _ptr(grid_masks), _ptr(status), _stream(stream))
+    _check(rc, "rs3_close_argmax")
+
+
+def rs3_seed_from_masks(masks, U: int, h: int, w: int, s: int, track, grid_masks, box_masks,
+                        stream=None):
+    rc = lib.rs3_seed_from_masks(_ptr(masks), U, h, w, s, _ptr(track), _ptr(grid_masks),
+                                 _ptr(box_masks), _stream(stream))
+    _check(rc, "rs3_seed_from_masks")

@@ -7,6 +7,12 @@ of the hot path for profilers:
 
 With --dense every cell is selected and nothing is write-pruned (rho = 1,
 all-ones masks): the unpruned comparison of the same kernels.
+
+    python -m paper_2608_22526_gb300.run_frames --workload sam2_8obj --close-argmax 3
+
+runs only the decoder-side call instead: rs3_close_argmax (the 9 x 9 closure
+per object, the palette argmax and down_s) on the workload's streams and
+objects, with 256 x 256 logits per 64 x 64 grid, the given number of times.
 """
 from __future__ import annotations
 
@@ -50,12 +56,33 @@ def run(workload: str, frames: int, dense: bool) -> Pipeline:
     return pipe
 
 
+def close_argmax(workload: str, launches: int) -> int:
+    from . import rs3
+    w = synth.WORKLOADS[workload]
+    h, wd = 4 * w.m, 4 * w.n
+    logits = _dev(synth.decoder_logits(np.random.default_rng(w.seed + 101), w.U, h, wd))
+    gs = torch.arange(0, w.U + 1, w.units_per_group, dtype=torch.int32, device="cuda")
+    pal = torch.empty((w.G, h, wd), dtype=torch.uint8, device="cuda")
+    grid = torch.empty((w.U, w.m, w.n), dtype=torch.uint8, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for _ in range(launches):
+        rs3.rs3_close_argmax(logits, gs, w.G, w.U, h, wd, 4, 4, pal, None, grid, status)
+    torch.cuda.synchronize()
+    return int(status.item())
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--workload", default="sam2_1obj", choices=sorted(synth.WORKLOADS))
     ap.add_argument("--frames", type=int, default=12)
     ap.add_argument("--dense", action="store_true")
+    ap.add_argument("--close-argmax", type=int, default=0, metavar="N",
+                    help="run rs3_close_argmax N times instead of the frames")
     args = ap.parse_args()
+    if args.close_argmax > 0:
+        st = close_argmax(args.workload, args.close_argmax)
+        print("status", st)
+        raise SystemExit(0 if st == 0 else 1)
     pipe = run(args.workload, args.frames, args.dense)
     print("status", pipe.status_code(), "count", pipe.count.tolist())
 

@@ -330,3 +330,51 @@ class Sequence:
 
 def random_bf16(rng: np.random.Generator, shape, scale: float = 1.0) -> np.ndarray:
     return f32_to_bf16_bits(rng.standard_normal(shape, dtype=np.float32) * np.float32(scale))
+
+
+# ----------------------------------------------------------------------------
+# Pixel-resolution inputs: decoder logits and seed masks
+# ----------------------------------------------------------------------------
+
+def decoder_logits(rng: np.random.Generator, n_obj: int, h: int, w: int,
+                   cov_lo: float = 0.02, cov_hi: float = 0.25,
+                   hole_rate: float = 0.01, speck_rate: float = 0.002) -> np.ndarray:
+    """Stand-in for a mask decoder's per-object logits [n_obj, h, w] fp32 at
+    its output resolution: a rotated ellipse per object (coverage drawn from
+    [cov_lo, cov_hi], objects may overlap and touch the border) with logits
+    |N(0,1)| + 0.5 inside and -(|N(0,1)| + 0.5) outside, then salt-and-pepper
+    noise -- isolated negative pixels inside ("holes", the artefact the paper's
+    closure removes) and isolated positive specks outside."""
+    out = np.empty((n_obj, h, w), dtype=np.float32)
+    for o in range(n_obj):
+        cov = rng.uniform(cov_lo, cov_hi)
+        aspect = rng.uniform(0.6, 1.6)
+        area = cov * h * w
+        a = math.sqrt(area * aspect / math.pi)
+        b = area / (math.pi * a)
+        cy, cx = rng.uniform(0.0, h), rng.uniform(0.0, w)
+        inside = ellipse_mask(h, w, cy, cx, a, b, rng.uniform(0.0, math.pi)).astype(bool)
+        mag = np.abs(rng.standard_normal((h, w), dtype=np.float32)) + np.float32(0.5)
+        lg = np.where(inside, mag, -mag)
+        holes = inside & (rng.random((h, w)) < hole_rate)
+        specks = ~inside & (rng.random((h, w)) < speck_rate)
+        lg[holes] = -lg[holes]
+        lg[specks] = -lg[specks]
+        out[o] = lg
+    return out
+
+
+def pixel_masks(rng: np.random.Generator, n_obj: int, h: int, w: int,
+                cov_lo: float = 0.02, cov_hi: float = 0.25) -> np.ndarray:
+    """First-frame object masks at pixel resolution [n_obj, h, w] uint8
+    (rotated ellipses, value 255 where set)."""
+    out = np.empty((n_obj, h, w), dtype=np.uint8)
+    for o in range(n_obj):
+        cov = rng.uniform(cov_lo, cov_hi)
+        aspect = rng.uniform(0.6, 1.6)
+        area = cov * h * w
+        a = math.sqrt(area * aspect / math.pi)
+        b = area / (math.pi * a)
+        cy, cx = rng.uniform(0.1 * h, 0.9 * h), rng.uniform(0.1 * w, 0.9 * w)
+        out[o] = ellipse_mask(h, w, cy, cx, a, b, rng.uniform(0.0, math.pi)) * np.uint8(255)
+    return out

@@ -114,3 +114,24 @@ def test_null_arguments_are_rejected_on_host(binding):
     assert lib.rs3_memory_readout(one, 1, 1, 4096, 1, 256, one, one, one, 1228, ctypes.byref(desc),
                                   None, None, one, 0.0, one, 1 << 30, one, None) == binding.RS3_EINVAL
     assert lib.rs3_write_keepset(None, one, 1, 8, 8, ctypes.byref(p), one, one, None) == binding.RS3_EINVAL
+
+
+def test_mask_calls_reject_bad_arguments_on_host(binding):
+    lib = binding.lib
+    one = ctypes.c_void_p(16)
+    E, U = binding.RS3_EINVAL, binding.RS3_EUNSUPPORTED
+    # logits, group_start, G, U, h, w, radius, s, palette, closed, grid, status, stream
+    assert lib.rs3_close_argmax(None, one, 1, 1, 64, 64, 4, 4, one, None, None, one, None) == E
+    assert lib.rs3_close_argmax(one, one, 1, 1, 64, 64, 4, 4, one, None, None, None, None) == E
+    assert lib.rs3_close_argmax(one, one, 1, 1, 64, 48, 4, 4, one, None, None, one, None) == U   # w % 32
+    assert lib.rs3_close_argmax(one, one, 1, 1, 64, 64, 9, 4, one, None, None, one, None) == U   # radius > 8
+    assert lib.rs3_close_argmax(one, one, 1, 1, 64, 64, -1, 4, one, None, None, one, None) == E
+    assert lib.rs3_close_argmax(one, one, 0, 1, 64, 64, 4, 4, one, None, None, one, None) == E
+    assert lib.rs3_close_argmax(one, one, 1, 1, 66, 64, 4, 4, None, None, one, one, None) == E   # h % s with grid
+    # masks, U, h, w, s, track, grid, box, stream
+    assert lib.rs3_seed_from_masks(None, 1, 64, 64, 16, one, None, None, None) == E
+    assert lib.rs3_seed_from_masks(one, 1, 64, 64, 16, None, None, None, None) == E
+    assert lib.rs3_seed_from_masks(one, 1, 64, 40, 8, one, None, None, None) == E      # w % 16
+    assert lib.rs3_seed_from_masks(one, 1, 64, 64, 24, one, None, None, None) == E     # w % s
+    assert lib.rs3_seed_from_masks(ctypes.c_void_p(17), 1, 64, 64, 16, one, None, None, None) == E
+    assert lib.rs3_seed_from_masks(one, 0, 64, 64, 16, one, None, None, None) == E

@@ -55,3 +55,11 @@ def test_workload_config_names_the_workload(name):
     assert cfg["workload"].startswith(name + ":")
     assert f"{w.m}x{w.n}" in cfg["workload"] and f"{w.frames} frames" in cfg["workload"]
     assert cfg["parallelism"] == "replicas x1"
+
+
+def test_close_argmax_work_closed_form():
+    w = synth.WORKLOADS["sam2_8obj"]
+    # 8 objects x 256^2 fp32 logits read, one 256^2 palette and 8 grid masks written
+    assert bench.close_argmax_work(w) == 8 * 256 * 256 * 4 + 256 * 256 + 8 * 64 * 64
+    w = synth.WORKLOADS["multistream"]
+    assert bench.close_argmax_work(w) == 48 * 384 * 384 * 4 + 16 * 384 * 384 + 48 * 96 * 96
