@@ -17,7 +17,7 @@
  *   closure + palette       Sec. 3.3 (9 x 9 closure per object, then argmax)
  *   down_s + seed box       Sec. 3.1 (pixel masks and boxes onto the grid)
  *
- * Readings where the paper is silent or ambiguous (documented in the design doc):
+ * Readings where the paper is silent or ambiguous:
  *   - dilate_r is a Chebyshev (square) dilation by r cells;
  *   - the streak counter is updated from the mask the selection consumes, and
  *     the fallback radius uses the incremented value (first empty frame -> r_s+1);
