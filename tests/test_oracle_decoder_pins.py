@@ -215,3 +215,28 @@ def test_seed_track_projects_the_pixel_box(s):
     assert list(orc.seed_track(M, s)) == [0, 0, 0, 0, 0, 0]
     M[h - 1, w - 1] = 1
     assert list(orc.seed_track(M, s)) == [(h - 1) // s, (w - 1) // s, (h - 1) // s, (w - 1) // s, 1, 0]
+
+
+# ---------------------------------------------------------------------------
+# the seeded pixel-resolution inputs the GPU tests and the benchmark share
+# ---------------------------------------------------------------------------
+
+def test_decoder_logits_are_seeded_and_shaped_like_the_recipe():
+    from paper_2608_22526_gb300 import synth
+    a = synth.decoder_logits(np.random.default_rng(5), 3, 64, 96)
+    b = synth.decoder_logits(np.random.default_rng(5), 3, 64, 96)
+    assert a.shape == (3, 64, 96) and a.dtype == np.float32 and np.array_equal(a, b)
+    assert np.all(np.abs(a) >= 0.5)                      # no logit on the threshold
+    cov = (a > 0).mean(axis=(1, 2))
+    assert np.all(cov > 0.005) and np.all(cov < 0.35)
+    # the salt-and-pepper holes are there for the closure to fill
+    closed = np.stack([orc.close(a[o] > 0, 64, 96, 4) for o in range(3)])
+    assert (closed.astype(int) - (a > 0)).sum() > 0
+
+
+def test_pixel_masks_are_seeded():
+    from paper_2608_22526_gb300 import synth
+    a = synth.pixel_masks(np.random.default_rng(8), 4, 128, 64)
+    b = synth.pixel_masks(np.random.default_rng(8), 4, 128, 64)
+    assert a.shape == (4, 128, 64) and a.dtype == np.uint8 and np.array_equal(a, b)
+    assert set(np.unique(a)) <= {0, 255} and np.all(a.reshape(4, -1).max(axis=1) == 255)
