@@ -167,7 +167,9 @@ rs3_status rs3_select_queries(const void *z, rs3_dtype dtype, int G, int m, int 
  *     library routine).
  *   - The first call on a device looks up the array's device address with
  *     that device current and caches it; make that first call before any
- *     stream capture.
+ *     stream capture.  The cache remembers the context the address belongs
+ *     to: after a device reset the next call looks the address up again, so
+ *     make that call before any capture too.
  *   - All calls on a device share the one array, and it keeps the previous
  *     call's contents (the call clears what must start at zero itself), so
  *     calls whose executions overlap on the GPU (different streams without
@@ -293,6 +295,9 @@ size_t rs3_readout_workspace_bytes(int U, int H, int d, int k_max, rs3_dtype dty
  *   workspace device, >= rs3_readout_workspace_bytes(...), 16-byte aligned
  * bf16: tensor-core path for d in {64, 128, 256}, fp32 accumulation.  fp32:
  * CUDA-core FFMA path for d % 16 == 0, d <= 256.
+ * Limits: U <= 4096, mn <= 16384; the work list holds fewer than 2^21
+ * entries (U * H * ceil(k_max / BM) plus one per SM, BM = 128 on the bf16
+ * path and 32 on the fp32 path), else RS3_EUNSUPPORTED.
  */
 rs3_status rs3_memory_readout(const void *q, rs3_dtype dtype, int G, int mn, int H, int d,
                               const int32_t *unit_group, const int32_t *idx,
@@ -300,6 +305,19 @@ rs3_status rs3_memory_readout(const void *q, rs3_dtype dtype, int G, int mn, int
                               const float *rope, const void *residual, void *out, float scale,
                               void *workspace, size_t workspace_bytes, int32_t *status,
                               rs3_stream_t stream);
+
+/*
+ * Time limit of every wait inside the readout kernels launched after this
+ * call, in nanoseconds of the GPU's global timer (default 1000000000, one
+ * second; 0 gives up at the first wait whose condition does not already
+ * hold).  A kernel whose wait runs out stops issuing work, lets its copies
+ * and matrix operations in flight complete, frees its tensor memory, latches
+ * RS3_ETIMEOUT into the call's status word and returns; the rows it did not
+ * finish hold unspecified values.  The setting is process-wide; it exists so
+ * that the timeout path can be exercised on purpose.  No paper counterpart.
+ */
+void rs3_set_wait_limit_ns(uint64_t ns);
+uint64_t rs3_get_wait_limit_ns(void);
 
 /*
  * The same readout in two phases, with the arguments of rs3_memory_readout
@@ -387,8 +405,10 @@ rs3_status rs3_close_argmax(const float *logits, const int32_t *group_start, int
  * tight pixel box of the set pixels, each corner divided by the encoder
  * stride s and rounded down, becomes the unit's tracker state ({y0, x0, y1,
  * x1} on the grid, valid 1, streak 0; an empty mask gives all zeros), so the
- * first rs3_select_queries call with an empty previous mask and bbox_mode, or
- * with box_masks as the previous mask, dilates down_s of the seed box.
+ * first rs3_select_queries call dilates down_s of the seed box: by r_s when
+ * box_masks is passed as the previous mask (Eq. 1), or by r_s + 1 when the
+ * previous mask is empty (Eq. 4's fallback, whose streak counter is already 1
+ * on that first empty frame).
  *   masks      device uint8 [U][h][w] (nonzero = set), 16-byte aligned
  *   track      device rs3_track [U], written
  *   grid_masks device uint8 [U][h/s][w/s] or NULL: down_s of the mask (cell

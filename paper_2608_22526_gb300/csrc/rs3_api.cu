@@ -3,6 +3,9 @@
 #include "rs3_internal.cuh"
 
 #include <cmath>
+#include <mutex>
+#include <utility>
+#include <vector>
 
 extern "C" void rs3_default_params(rs3_params *p)
 {
@@ -55,3 +58,26 @@ int rs3_sm_count()
 }
 
 bool rs3_aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+rs3_status rs3_kernel_smem(const void *kernel, size_t bytes)
+{
+    if (bytes <= 48 * 1024) return RS3_OK;     // the default limit
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return RS3_ECUDA;
+    static std::mutex mu;
+    static std::vector<std::pair<std::pair<const void *, int>, size_t>> done;   // (kernel, device) -> bytes
+    std::lock_guard<std::mutex> lock(mu);
+    for (auto &e : done)
+        if (e.first.first == kernel && e.first.second == dev) {
+            if (e.second >= bytes) return RS3_OK;
+            if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes) !=
+                cudaSuccess)
+                return RS3_ECUDA;
+            e.second = bytes;
+            return RS3_OK;
+        }
+    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes) != cudaSuccess)
+        return RS3_ECUDA;
+    done.push_back({{kernel, dev}, bytes});
+    return RS3_OK;
+}

@@ -136,3 +136,7 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
 // Host helpers implemented in rs3_api.cu
 int rs3_sm_count();
 bool rs3_aligned16(const void *p);
+// Raises `kernel`'s dynamic shared-memory limit on the current device to at
+// least `bytes` (once per kernel and device; safe to call from several host
+// threads).  RS3_ECUDA when the runtime refuses.
+rs3_status rs3_kernel_smem(const void *kernel, size_t bytes);

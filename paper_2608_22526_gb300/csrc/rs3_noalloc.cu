@@ -10,6 +10,8 @@
 // scratch lives in a fixed device array compiled into the library.
 #include "rs3_internal.cuh"
 
+#include <cuda.h>
+
 #include <mutex>
 
 // 8 MiB of scratch, held by every GPU that loads the library until the process
@@ -22,21 +24,54 @@ namespace {
 
 std::mutex g_setup_mutex;
 void *g_scratch_ptr[64] = {nullptr};
+unsigned long long g_scratch_ctx[64] = {0};   // id of the context the address belongs to
+
+typedef CUresult (*ctx_get_current_fn)(CUcontext *);
+typedef CUresult (*ctx_get_id_fn)(CUcontext, unsigned long long *);
+
+// Id of the calling thread's current context (0 when it cannot be asked).  A
+// device reset, or a new primary context, gives the array a new address; the
+// id tells the cached address from the current one.
+unsigned long long current_context_id()
+{
+    static ctx_get_current_fn get_cur = nullptr;
+    static ctx_get_id_fn get_id = nullptr;
+    static bool looked = false;
+    if (!looked) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_cur = reinterpret_cast<ctx_get_current_fn>(p);
+        p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<ctx_get_id_fn>(p);
+        looked = true;
+    }
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (!get_cur || !get_id || get_cur(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+    return id;
+}
 
 // Device address of the scratch array on the current device.  In host code
 // the array's name is only a host-side stand-in, so the address is asked from
-// the runtime once per device (with that device current) and cached.
+// the runtime with the device current, and cached per device together with
+// the id of the context it belongs to (asked again when that id changes).
 rs3_status scratch_for_current_device(void **out)
 {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return RS3_ECUDA;
     if (dev < 0 || dev >= 64) return RS3_EUNSUPPORTED;
     std::lock_guard<std::mutex> lock(g_setup_mutex);
-    if (g_scratch_ptr[dev] == nullptr) {
+    const unsigned long long ctx = current_context_id();
+    if (g_scratch_ptr[dev] == nullptr || (ctx != 0 && ctx != g_scratch_ctx[dev])) {
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, rs3_noalloc_scratch) != cudaSuccess || p == nullptr)
             return RS3_ECUDA;
         g_scratch_ptr[dev] = p;
+        g_scratch_ctx[dev] = current_context_id();
     }
     *out = g_scratch_ptr[dev];
     return RS3_OK;

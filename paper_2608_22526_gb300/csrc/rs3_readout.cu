@@ -19,6 +19,7 @@
 // rs3_memory_readout_attend / _merge issue one each.
 #include "rs3_internal.cuh"
 
+#include <atomic>
 #include <cmath>
 
 #include "rs3_readout_common.cuh"
@@ -593,6 +594,13 @@ ReadoutLayout readout_layout(int U, int H, int d, int k_max, int BM, int grid)
 
 }  // namespace
 
+namespace {
+std::atomic<uint64_t> g_wait_ns{1000000000ull};
+}
+
+extern "C" void rs3_set_wait_limit_ns(uint64_t ns) { g_wait_ns.store(ns); }
+extern "C" uint64_t rs3_get_wait_limit_ns(void) { return g_wait_ns.load(); }
+
 ReadoutPath choose_readout_path(rs3_dtype dtype, int d)
 {
     ReadoutPath p;
@@ -639,6 +647,8 @@ rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, in
         return RS3_EINVAL;
     const ReadoutPath p = choose_readout_path(dtype, d);
     const ReadoutLayout L = readout_layout(bank->U, H, d, k_max, p.BM, p.grid);
+    // the plan packs its per-CTA counts into PK_SHIFT-bit fields
+    if (L.max_items >= PK_MASK || L.max_slots >= PK_MASK || L.max_combine >= PK_MASK) return RS3_EUNSUPPORTED;
     if (workspace_bytes < L.total) return RS3_ECAPACITY;
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     a->q = q;
@@ -677,6 +687,7 @@ rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, in
     a->cta_items = reinterpret_cast<int32_t *>(ws + L.cta_items);
     const float sc = scale > 0.f ? scale : 1.0f / sqrtf((float)d);
     a->scale_log2 = sc * 1.4426950408889634f;
+    a->wait_ns = g_wait_ns.load();
     a->header = reinterpret_cast<ReadoutHeader *>(ws + L.header);
     a->ranges = reinterpret_cast<RangeSet *>(ws + L.ranges);
     a->items = reinterpret_cast<WorkItem *>(ws + L.items);
@@ -705,26 +716,16 @@ rs3_status launch_attend(const ReadoutArgs &a, const ReadoutPath &p, rs3_dtype d
     }
     // plan shared memory: unit slot bases and widths, slice bounds, per-CTA counts, unit tiles
     const size_t plan_smem = ((size_t)(2 * a.U + 1) + 2 * (size_t)(a.grid_ctas + 1)) * 8 + (size_t)a.U * 4;
-    static size_t plan_attr = 0;
-    if (plan_smem > 48 * 1024 && plan_smem > plan_attr) {
-        if (cudaFuncSetAttribute(k_plan, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan_smem) !=
-            cudaSuccess)
-            return RS3_EUNSUPPORTED;
-        plan_attr = plan_smem;
-    }
+    if (rs3_kernel_smem((const void *)k_plan, plan_smem) != RS3_OK) return RS3_EUNSUPPORTED;
     launch_pdl(k_plan, dim3(1), dim3(PLAN_THREADS), plan_smem, st, a);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     if (p.kind == 1) return rs3_launch_tc_readout(a, st);
     const size_t smem = (size_t)2 * SIMT_BN * a.d * sizeof(float);
     const int threads = 2 * a.d;
     const int64_t blocks = a.grid_ctas;
-    static bool attr_done = false;
-    if (!attr_done) {
-        const int most = 2 * SIMT_BN * 256 * (int)sizeof(float);
-        cudaFuncSetAttribute(k_readout_simt<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
-        cudaFuncSetAttribute(k_readout_simt<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
-        attr_done = true;
-    }
+    if (rs3_kernel_smem(dtype == RS3_BF16 ? (const void *)k_readout_simt<uint16_t>
+                                          : (const void *)k_readout_simt<float>, smem) != RS3_OK)
+        return RS3_ECUDA;
     if (dtype == RS3_BF16)
         launch_pdl(k_readout_simt<uint16_t>, dim3((unsigned)blocks), dim3(threads), smem, st, a);
     else

@@ -29,7 +29,8 @@
 // TMEM (512 columns): O in [0, d), S_0 / S_1 from S_COL, Q at Q_COL.
 // Shapes: d = 256 and d = 128 use 64-key tiles, d = 64 128-key tiles; K and V
 // rings fill what shared memory leaves after the three P buffers.
-// Every mbarrier wait is bounded (1 s of %globaltimer): on expiry the CTA
+// Every mbarrier wait is bounded (a launch parameter, 1 s of %globaltimer by
+// default): on expiry the CTA
 // raises an abort flag, drains its copies and MMAs, frees TMEM and the launch
 // latches RS3_ETIMEOUT.
 #include "rs3_readout_common.cuh"
@@ -213,6 +214,7 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    const uint64_t wait_ns = a.wait_ns;
     // the set-up above touches no global memory; the plan is read after the
     // previous kernel of the stream has completed
     pdl_wait();
@@ -235,7 +237,7 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             const RangeSet *rs = a.ranges + w.u;
             for (int t = w.tile_begin; t < w.tile_end; ++t, ++cnt) {
                 const uint32_t st = cnt % nst, ph = (cnt / nst) & 1u;
-                if (!mbar_wait(BAR(b_empty + st), ph ^ 1u, abort_flag)) goto producer_done;
+                if (!mbar_wait(BAR(b_empty + st), ph ^ 1u, abort_flag, wait_ns)) goto producer_done;
                 int64_t row0;
                 int nvalid;
                 tile_rows(rs, t, BN, row0, nvalid);
@@ -268,12 +270,12 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             const WorkItem w = a.items[it];
             const int n = w.tile_end - w.tile_begin;
             if (n <= 0) continue;
-            if (!mbar_wait(BAR(C::B_QFULL), icnt & 1u, abort_flag)) { ok = false; break; }
+            if (!mbar_wait(BAR(C::B_QFULL), icnt & 1u, abort_flag, wait_ns)) { ok = false; break; }
             ++icnt;
             for (int j = 0; j < n; ++j) {
                 const uint32_t t = tcnt + (uint32_t)j, st = t % KSTK, b = t & 1u;
-                if (!mbar_wait(BAR(C::B_SFREE + b), ((t >> 1) & 1u) ^ 1u, abort_flag)) { ok = false; break; }
-                if (!mbar_wait(BAR(C::B_KFULL + st), (t / KSTK) & 1u, abort_flag)) { ok = false; break; }
+                if (!mbar_wait(BAR(C::B_SFREE + b), ((t >> 1) & 1u) ^ 1u, abort_flag, wait_ns)) { ok = false; break; }
+                if (!mbar_wait(BAR(C::B_KFULL + st), (t / KSTK) & 1u, abort_flag, wait_ns)) { ok = false; break; }
                 tc_fence_after();
                 const uint64_t dks = dk0 + st * STAGE16;
                 const uint32_t dst = tmem + C::S_COL + (uint32_t)BN * b;
@@ -306,8 +308,8 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             if (n <= 0) continue;
             for (int j = 0; j < n; ++j) {
                 const uint32_t tj = tcnt + (uint32_t)j, pb = tj % C::NPB, st = tj % KSTV;
-                if (!mbar_wait(BAR(C::B_PFULL + pb), (tj / C::NPB) & 1u, abort_flag)) { ok = false; break; }
-                if (!mbar_wait(BAR(C::B_VFULL + st), (tj / KSTV) & 1u, abort_flag)) { ok = false; break; }
+                if (!mbar_wait(BAR(C::B_PFULL + pb), (tj / C::NPB) & 1u, abort_flag, wait_ns)) { ok = false; break; }
+                if (!mbar_wait(BAR(C::B_VFULL + st), (tj / KSTV) & 1u, abort_flag, wait_ns)) { ok = false; break; }
                 tc_fence_after();
                 const uint64_t dvs = dv0 + st * STAGE16, dps = dp0 + pb * PBUF16;
 #pragma unroll
@@ -399,7 +401,7 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             float m_run = -INFINITY, l_part = 0.f;
             for (int j = 0; j < n; ++j) {
                 const uint32_t tj = tcnt + (uint32_t)j, b = tj & 1u;
-                const bool okw = __all_sync(0xffffffffu, mbar_wait(BAR(C::B_SFULL + b), (tj >> 1) & 1u, abort_flag));
+                const bool okw = __all_sync(0xffffffffu, mbar_wait(BAR(C::B_SFULL + b), (tj >> 1) & 1u, abort_flag, wait_ns));
                 int nvt = 0;
                 {
                     int t = w.tile_begin + j;
@@ -464,7 +466,7 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
                             // barrier takes every slice out
                             const uint32_t tp = tj - 1u;
                             if (__all_sync(0xffffffffu, mbar_wait(BAR(C::B_PVDONE + tp % C::NPB),
-                                                                  (tp / C::NPB) & 1u, abort_flag))) {
+                                                                  (tp / C::NPB) & 1u, abort_flag, wait_ns))) {
                                 tc_fence_after();
 #pragma unroll 1
                                 for (int c16 = 0; c16 < OCOLS / 16; ++c16) {
@@ -489,7 +491,7 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
                 // PV_{j-3}.  On a timeout the store is skipped and the next
                 // barrier takes every slice out.
                 if (__all_sync(0xffffffffu, mbar_wait(BAR(C::B_PVDONE + tj % C::NPB),
-                                                      ((tj / C::NPB) & 1u) ^ 1u, abort_flag))) {
+                                                      ((tj / C::NPB) & 1u) ^ 1u, abort_flag, wait_ns))) {
                     const uint32_t pbase = sP + (tj % C::NPB) * C::PBYTES;
 #pragma unroll
                     for (int cc = 0; cc < PCOLS / 4; ++cc) {
@@ -508,7 +510,7 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
             if (n > 0) {
                 const uint32_t tlast = tcnt + (uint32_t)n - 1u;
                 const bool okw = __all_sync(0xffffffffu, mbar_wait(BAR(C::B_PVDONE + tlast % C::NPB),
-                                                                   (tlast / C::NPB) & 1u, abort_flag));
+                                                                   (tlast / C::NPB) & 1u, abort_flag, wait_ns));
                 float *redl = red + (2 * NSPLIT) * BM;
                 redl[h * BM + r] = l_part;
                 if (!bar_and(bar_id, bar_n, okw)) { ok = false; break; }
@@ -641,13 +643,7 @@ bool make_kv_map(CUtensorMap *m, const void *store, int64_t D, int64_t rows, int
 template <int DH>
 rs3_status launch(const ReadoutArgs &a, cudaStream_t st)
 {
-    static bool attr = false;
-    if (!attr) {
-        if (cudaFuncSetAttribute(k_readout_tc<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<DH>::SMEM) !=
-            cudaSuccess)
-            return RS3_ECUDA;
-        attr = true;
-    }
+    if (rs3_kernel_smem((const void *)k_readout_tc<DH>, Cfg<DH>::SMEM) != RS3_OK) return RS3_ECUDA;
     const int64_t rows = (int64_t)a.U * a.rows_per_unit;
     if (rows >= (int64_t)1 << 31) return RS3_EUNSUPPORTED;
     CUtensorMap mk, mv;

@@ -505,11 +505,7 @@ extern "C" rs3_status rs3_select_queries(const void *z, rs3_dtype dtype, int G, 
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
 
     const size_t smem_sel = (size_t)mn * 4;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, RS3_MAX_MN * 4);
-        attr_set = true;
-    }
+    if (rs3_kernel_smem((const void *)k_select, smem_sel) != RS3_OK) return RS3_ECUDA;
     launch_pdl(k_select, dim3(U), dim3(1024), smem_sel, st, prior, need, energy, unit_group, G, mn, p->union_mode,
                                         (int)k, idx, count);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;

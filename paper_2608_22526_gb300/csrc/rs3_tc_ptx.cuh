@@ -8,7 +8,7 @@
 
 namespace tc {
 
-constexpr uint64_t WAIT_LIMIT_NS = 1000000000ull;   // a wait gives up after 1 s
+constexpr uint64_t DRAIN_LIMIT_NS = 1000000000ull;  // a drain of work in flight gives up after 1 s
 
 
 // ---------------------------------------------------------------------------
@@ -55,27 +55,31 @@ __device__ __forceinline__ uint64_t gtimer()
 }
 
 // Waits for the phase with parity `parity` to complete; gives up (and raises
-// the CTA's abort flag) after WAIT_LIMIT_NS, or at once if the flag is up.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag)
+// the CTA's abort flag) once more than `limit_ns` have passed, or at once if
+// the flag is up.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag,
+                                          uint64_t limit_ns)
 {
     if (mbar_try(bar, parity)) return true;
     const uint64_t t0 = gtimer();
     while (true) {
         if (mbar_try(bar, parity)) return true;
         if (*abort_flag) return false;
-        if (gtimer() - t0 > WAIT_LIMIT_NS) {
+        if (gtimer() - t0 >= limit_ns) {
             *abort_flag = 1;
             return false;
         }
     }
 }
 
-// Bounded wait that ignores the abort flag (used to drain work in flight).
+// Bounded wait that ignores the abort flag, for draining copies and matrix
+// operations already issued (they complete on their own; the limit only
+// guards against a broken device).
 __device__ __forceinline__ void mbar_drain(uint32_t bar, uint32_t parity)
 {
     const uint64_t t0 = gtimer();
     while (!mbar_try(bar, parity))
-        if (gtimer() - t0 > WAIT_LIMIT_NS) return;
+        if (gtimer() - t0 > DRAIN_LIMIT_NS) return;
 }
 
 __device__ __forceinline__ void prefetch_l2(const void *p)

@@ -72,6 +72,8 @@ SIGNATURES = {
                                 ctypes.c_float, _P, _SZ, _P, _P]),
     "rs3_memory_readout_merge": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P, _P, _P, _P,
                                 ctypes.c_float, _P, _SZ, _P, _P]),
+    "rs3_set_wait_limit_ns": (None, [ctypes.c_uint64]),
+    "rs3_get_wait_limit_ns": (ctypes.c_uint64, []),
     "rs3_write_keepset": (_I, [_P, _P, _I, _I, _I, _P, _P, _P, _P]),
     "rs3_close_argmax": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
     "rs3_seed_from_masks": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P]),
@@ -290,3 +292,11 @@ def rs3_seed_from_masks(masks, U: int, h: int, w: int, s: int, track, grid_masks
     rc = lib.rs3_seed_from_masks(_ptr(masks), U, h, w, s, _ptr(track), _ptr(grid_masks),
                                  _ptr(box_masks), _stream(stream))
     _check(rc, "rs3_seed_from_masks")
+
+
+def rs3_set_wait_limit_ns(ns: int):
+    lib.rs3_set_wait_limit_ns(int(ns))
+
+
+def rs3_get_wait_limit_ns() -> int:
+    return int(lib.rs3_get_wait_limit_ns())

@@ -332,6 +332,37 @@ def random_bf16(rng: np.random.Generator, shape, scale: float = 1.0) -> np.ndarr
     return f32_to_bf16_bits(rng.standard_normal(shape, dtype=np.float32) * np.float32(scale))
 
 
+def ternary_grid(rng: np.random.Generator, G: int, mn: int, C: int, p_nonzero: float,
+                 dtype: str = "bf16") -> np.ndarray:
+    """Token grids whose channels are -1, 0 or +1 (nonzero with probability
+    p_nonzero, either sign equally likely).  Every squared norm is an integer
+    in [0, C], so many cells share one, which puts equal keys at the k-th
+    place of a top-k.  Returns bf16 bits or fp32 [G, mn, C]."""
+    mag = (rng.random((G, mn, C)) < p_nonzero).astype(np.float32)
+    sign = np.where(rng.random((G, mn, C)) < 0.5, -1.0, 1.0).astype(np.float32)
+    z = mag * sign
+    return f32_to_bf16_bits(z) if dtype == "bf16" else z
+
+
+def permuted_rows(rng: np.random.Generator, G: int, mn: int, C: int,
+                  dtype: str = "bf16") -> np.ndarray:
+    """Token grids whose rows are permutations of one N(0,1) vector per grid:
+    every cell of a grid has the same multiset of channel values."""
+    base = rng.standard_normal((G, C), dtype=np.float32)
+    z = np.empty((G, mn, C), dtype=np.float32)
+    for g in range(G):
+        z[g] = base[g][rng.permuted(np.tile(np.arange(C), (mn, 1)), axis=1)]
+    return f32_to_bf16_bits(z) if dtype == "bf16" else z
+
+
+def cell_subset_masks(rng: np.random.Generator, U: int, mn: int, sizes) -> np.ndarray:
+    """Masks [U, mn] with exactly sizes[u] set cells each, at random positions."""
+    M = np.zeros((U, mn), np.uint8)
+    for u in range(U):
+        M[u, rng.choice(mn, size=int(sizes[u]), replace=False)] = 1
+    return M
+
+
 # ----------------------------------------------------------------------------
 # Pixel-resolution inputs: decoder logits and seed masks
 # ----------------------------------------------------------------------------

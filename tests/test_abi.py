@@ -135,3 +135,29 @@ def test_mask_calls_reject_bad_arguments_on_host(binding):
     assert lib.rs3_seed_from_masks(one, 1, 64, 64, 24, one, None, None, None) == E     # w % s
     assert lib.rs3_seed_from_masks(ctypes.c_void_p(17), 1, 64, 64, 16, one, None, None, None) == E
     assert lib.rs3_seed_from_masks(one, 0, 64, 64, 16, one, None, None, None) == E
+
+
+def test_oversized_readout_plan_is_refused(binding):
+    """The readout's work list packs per-CTA counts into 21-bit fields: a
+    request whose list could reach 2^21 entries (4096 units, k_max 16384 on
+    the fp32 path: 4096 x 512 query tiles) is refused on the host with
+    RS3_EUNSUPPORTED; a small request with the same descriptor shape gets as
+    far as the workspace-size check."""
+    lib = binding.lib
+    one = ctypes.c_void_p(16)
+
+    def bank(U):
+        b = binding.BankDesc()
+        b.U, b.H, b.d, b.D, b.dtype, b.mn = U, 1, 64, 64, 0, 16384
+        b.n_cond, b.window, b.max_frames, b.n_ptr = 0, -1, 4, 0
+        b.pinned_cap, b.ring_cap, b.rows_per_unit, b.meta_stride = 0, 64, 64, 8 * 24
+        b.k_store = b.v_store = b.meta = one
+        b.magic = 0x52533342           # what rs3_bank_init stores
+        return b
+
+    big, small = bank(4096), bank(8)
+    args = lambda b, ws: (one, 0, 1, 16384, 1, 64, one, one, one, 16384, ctypes.byref(b), None, None,
+                          one, 0.0, one, ws, one, None)
+    assert lib.rs3_memory_readout(*args(big, 1 << 62)) == binding.RS3_EUNSUPPORTED
+    assert lib.rs3_memory_readout_attend(*args(big, 1 << 62)) == binding.RS3_EUNSUPPORTED
+    assert lib.rs3_memory_readout(*args(small, 16)) == binding.RS3_ECAPACITY

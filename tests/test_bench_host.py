@@ -42,10 +42,25 @@ def test_traffic_key_ignores_comments_not_code(tmp_path, monkeypatch):
     assert bench.readout_source_hash() != h0
 
 
-def test_traffic_record_matches_the_committed_sources():
-    """profiles/traffic.json was taken on the readout kernel as committed."""
-    rec = bench._traffic_record(synth.WORKLOADS["sam2_1obj"])
-    assert rec is not None and rec > 0
+def test_traffic_record_is_used_only_with_its_sources(tmp_path, monkeypatch):
+    """A stored DRAM-traffic figure is reported only while the readout
+    sources hash to the key it was stored with; otherwise the bench reports
+    null."""
+    import json
+    w = synth.WORKLOADS["sam2_8obj"]
+    src = os.path.join(ROOT, "paper_2608_22526_gb300", "csrc")
+    dst = tmp_path / "paper_2608_22526_gb300" / "csrc"
+    dst.mkdir(parents=True)
+    for f in ("rs3_readout.cu", "rs3_readout_tc.cu", "rs3_readout_common.cuh", "rs3_tc_ptx.cuh"):
+        shutil.copy(os.path.join(src, f), dst / f)
+    (tmp_path / "profiles").mkdir()
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    rec = {"source_hash": bench.readout_source_hash(), "per_launch_bytes": {w.name: 12345}}
+    (tmp_path / "profiles" / "traffic.json").write_text(json.dumps(rec))
+    assert bench._traffic_record(w) == 12345
+    rec["source_hash"] = "0" * 16
+    (tmp_path / "profiles" / "traffic.json").write_text(json.dumps(rec))
+    assert bench._traffic_record(w) is None
 
 
 @pytest.mark.parametrize("name", sorted(synth.WORKLOADS))

@@ -180,3 +180,54 @@ def test_ragged_counts_across_units_and_tiles():
     w = synth.Workload("ragged", 10, 48, 48, 1, 128, "bf16", 1, 5, 12, 0.01, 0.5, 1, 3, 5)
     from tests._harness import run_lockstep
     run_lockstep(w, check_frames={1, 5, 11}, residual_mode="inplace")
+
+
+def test_readout_wait_limit_runs_out_and_the_context_stays_usable():
+    """Every wait of the tensor-core readout has a time limit.  With the limit
+    at 0 ns the waits give up at once: the launch returns, latches
+    RS3_ETIMEOUT, and frees its tensor memory (the following launches on
+    every SM allocate it again); later calls with the default limit are
+    correct against the oracle."""
+    from tests._harness import check_fused
+    w = synth.scaled(W["sam2_1obj"], frames=3)
+    pipe = Pipeline(w)
+    seq = synth.Sequence(w)
+    kn, vn = seq.kv_new(0)
+    pipe.commit(to_dev(kn), to_dev(vn), to_dev(seq.masks(0)), 1)
+    kp, vp = seq.pointers()
+    pipe.set_pointers(to_dev(kp), to_dev(vp))
+    z = seq.z(1)
+    pipe.select(to_dev(z), to_dev(seq.masks(0)))
+    torch.cuda.synchronize()
+    assert rs3.rs3_get_wait_limit_ns() == 10 ** 9
+    x = z[w.unit_group()]
+    rs3.rs3_set_wait_limit_ns(0)
+    try:
+        for _ in range(2):
+            res = to_dev(x)
+            pipe.readout(to_dev(z), res, res)
+        torch.cuda.synchronize()
+    finally:
+        rs3.rs3_set_wait_limit_ns(10 ** 9)
+    assert pipe.status_code() == rs3.RS3_ETIMEOUT
+    pipe.status.zero_()
+    # the oracle's view of the bank and keep-set
+    ob = orc.OracleBank(w.U, w.D, w.dtype, w.mn, w.n_cond, w.window, pipe.bank.ring_cap,
+                        pipe.bank.max_frames, w.n_ptr)
+    ob.commit(kn, vn, seq.masks(0), 1)
+    ob.set_pointers(kp, vp)
+    track = np.zeros((w.U, 6), np.int32)
+    sel = orc.select(z, w.dtype, seq.masks(0), w.unit_group(), track, w.m, w.n, w.rho, w.r_s, w.c,
+                     w.union_mode)
+    keep = sel.keep(0)
+    K, V = ob.kv(0)
+    A = orc.readout(z[0], w.dtype, w.H, w.d, keep, K, V, w.dtype, threads=8)
+    rep = Report()
+    for _ in range(3):
+        res = to_dev(x)
+        pipe.readout(to_dev(z), res, res)
+        out = to_host(res)
+        check_fused(w.dtype, out[0][keep], x[0][keep], A, rep, "after the timeout")
+        others = np.setdiff1d(np.arange(w.mn), keep)
+        assert np.array_equal(out[0][others], x[0][others])
+    assert pipe.status_code() == 0
