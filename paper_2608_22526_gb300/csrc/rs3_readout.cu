@@ -73,34 +73,46 @@ __device__ RangeSet unit_ranges(const ReadoutArgs &a, int u, int cnt)
     return rs;
 }
 
-// exclusive scan of an int64 per thread, returns offset; *total = block total
-__device__ int64_t block_scan64(int64_t v, int64_t *total)
+// Exclusive block scan of an (int64, int32) pair per thread; returns the
+// offsets and writes the block totals.
+__device__ void block_scan_pair(int64_t v, int32_t g, int64_t &off_v, int32_t &off_g, int64_t &tot_v,
+                                int32_t &tot_g)
 {
-    __shared__ int64_t s_part[32];
-    __shared__ int64_t s_tot;
+    __shared__ int64_t s_pv[32];
+    __shared__ int32_t s_pg[32];
+    __shared__ int64_t s_tv;
+    __shared__ int32_t s_tg;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-    int64_t incl = v;
+    int64_t iv = v;
+    int32_t ig = g;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-        const int64_t t = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += t;
+        const int64_t tv = __shfl_up_sync(0xffffffffu, iv, o);
+        const int32_t tg = __shfl_up_sync(0xffffffffu, ig, o);
+        if (lane >= o) { iv += tv; ig += tg; }
     }
-    if (lane == 31) s_part[warp] = incl;
+    if (lane == 31) { s_pv[warp] = iv; s_pg[warp] = ig; }
     __syncthreads();
     if (threadIdx.x == 0) {
-        int64_t run = 0;
+        int64_t rv = 0;
+        int32_t rg = 0;
         for (int w = 0; w < nw; ++w) {
-            const int64_t t = s_part[w];
-            s_part[w] = run;
-            run += t;
+            const int64_t tv = s_pv[w];
+            const int32_t tg = s_pg[w];
+            s_pv[w] = rv;
+            s_pg[w] = rg;
+            rv += tv;
+            rg += tg;
         }
-        s_tot = run;
+        s_tv = rv;
+        s_tg = rg;
     }
     __syncthreads();
-    const int64_t off = s_part[warp] + incl - v;
-    *total = s_tot;
+    off_v = s_pv[warp] + iv - v;
+    off_g = s_pg[warp] + ig - g;
+    tot_v = s_tv;
+    tot_g = s_tg;
     __syncthreads();
-    return off;
 }
 
 // Stream-K plan.  Group g = (unit u, query tile qt, head h) owns
@@ -108,22 +120,38 @@ __device__ int64_t block_scan64(int64_t v, int64_t *total)
 // the unit's bank): OV leading slots stand for the fixed cost of starting a
 // piece of work (loading the query rows, the epilogue), so a CTA whose slice
 // starts groups gets fewer tiles, and the T_u tile slots follow.  CTA b of P
-// takes slots [sb[b], sb[b+1]) with sb[b] = b W / P; its slice is cut at group
+// takes slots [sb(b), sb(b+1)) with sb(b) = b W / P; its slice is cut at group
 // boundaries into items, each the tiles of the group its part covers.  A group
-// whose tiles a slice boundary cuts is split: its pieces write partials to
-// consecutive slots (CTA order) and the CTA holding its first tile emits the
-// combine entry.  A group with no tiles (empty bank) is one item with no
-// tiles, emitted where its first slot lies, so its rows are still written.
+// with no tiles (empty bank) is one item with no tiles, emitted where its first
+// slot lies, so its rows are still written.
+//
+// Indexing without a scan over the slices: the piece of group G (linear index
+// over all units' groups) in slice b is item G + b.  Each group's pieces lie in
+// consecutive slices and the groups follow each other along the axis, so the
+// indices are unique and a slice's items are consecutive.  Only a slice's first
+// item can be cut at its start and only its last at its end, so a split piece
+// takes partial slot 2b (the slice's first item) or 2b + 1 (its last); a split
+// group's later pieces are each the first item of their slice.  The slice that
+// holds a split group's first tile emits the group's merge entry (the entries
+// are packed in any order).
 struct PlanView {
     const int64_t *tb;   // [U+1] first linear slot of each unit
     const int64_t *wg;   // [U]   slots per group of each unit
     const int32_t *nt;   // [U]   key tiles of each unit
-    const int64_t *sb;   // [P+1] first slot of each slice
+    const int32_t *gb;   // [U+1] first linear group of each unit
     int U, H;
     int64_t W;
     int P;
     int ov;              // leading slots of a group (the start-up cost)
 };
+
+// b W / P; in 32 bits when b W cannot reach 2^32 (W < 2^22, b < 1024)
+__device__ __forceinline__ int64_t slice_start(const PlanView &v, int b)
+{
+    if (v.P <= 0) return 0;
+    if (v.W < ((int64_t)1 << 22) && b < 1024) return (int64_t)((uint32_t)b * (uint32_t)v.W / (uint32_t)v.P);
+    return (int64_t)b * v.W / v.P;
+}
 
 __device__ __forceinline__ void locate(const PlanView &v, int64_t x, int &u, int &gl, int64_t &off)
 {
@@ -134,17 +162,24 @@ __device__ __forceinline__ void locate(const PlanView &v, int64_t x, int &u, int
     }
     u = lo;
     const int64_t rel = x - v.tb[u];
-    gl = (int)(rel / v.wg[u]);
+    if (v.W < ((int64_t)1 << 22)) {
+        gl = (int)((uint32_t)rel / (uint32_t)v.wg[u]);
+    } else {
+        gl = (int)(rel / v.wg[u]);
+    }
     off = rel - (int64_t)gl * v.wg[u];
 }
 
-// Walks CTA b's slice; with write == false only counts items, partial items
-// and combine entries.
-__device__ void plan_slice(const ReadoutArgs &a, const PlanView &v, int b, bool write, int64_t item0,
-                           int64_t slot0, int64_t comb0, int &n_items, int &n_part, int &n_comb)
+// Writes slice b's items and its item range; returns its merge entry in c
+// (nsplit 0: none) and its partial pieces in n_part.
+__device__ void plan_slice(const ReadoutArgs &a, const PlanView &v, int b, int &n_part, CombineItem &c)
 {
-    n_items = n_part = n_comb = 0;
-    const int64_t lo = v.sb[b], hi = v.sb[b + 1];
+    const int64_t lo = slice_start(v, b), hi = slice_start(v, b + 1);
+    int64_t first = -1, last = -1;
+    c.u = c.h = c.qt = c.slot0 = c.nsplit = 0;
+    c.pad[0] = b;
+    c.pad[1] = c.pad[2] = 0;
+    n_part = 0;
     for (int64_t x = lo; x < hi;) {
         int u, gl;
         int64_t off;
@@ -158,46 +193,33 @@ __device__ void plan_slice(const ReadoutArgs &a, const PlanView &v, int b, bool 
         const bool emit = nt > 0 ? t1 > t0 : off == 0;
         if (emit) {
             const bool whole = t0 == 0 && t1 == nt;
-            if (write) {
-                WorkItem w;
-                w.u = u; w.qt = gl / v.H; w.h = gl % v.H; w.split = 0;
-                w.tile_begin = (int32_t)t0;
-                w.tile_end = (int32_t)t1;
-                w.slot = whole ? -1 : (int32_t)(slot0 + n_part);
-                w.pad = 0;
-                a.items[item0 + n_items] = w;
-                if (!whole && t0 == 0) {
-                    // first piece of a split group: the last slice it reaches is
-                    // the last e with sb[e] <= the group's last slot
-                    const int64_t gend = x - off + wg - 1;
-                    int lo_e = b, hi_e = v.P;              // sb[lo_e] <= gend < sb[hi_e]
-                    while (hi_e - lo_e > 1) {
-                        const int mid = (lo_e + hi_e) >> 1;
-                        if (v.sb[mid] <= gend) lo_e = mid; else hi_e = mid;
-                    }
-                    CombineItem c;
-                    c.u = u; c.h = w.h; c.qt = w.qt;
-                    c.slot0 = (int32_t)(slot0 + n_part);
-                    c.nsplit = lo_e - b + 1;
-                    c.pad[0] = c.pad[1] = c.pad[2] = 0;
-                    a.combine[comb0 + n_comb] = c;
-                }
-            }
-            ++n_items;
-            if (!whole) {
-                if (t0 == 0) ++n_comb;
-                ++n_part;
+            const int64_t idx = (int64_t)v.gb[u] + gl + b;
+            WorkItem w;
+            w.u = u; w.qt = gl / v.H; w.h = gl % v.H; w.split = 0;
+            w.tile_begin = (int32_t)t0;
+            w.tile_end = (int32_t)t1;
+            w.slot = whole ? -1 : 2 * b + (first < 0 ? 0 : 1);
+            w.pad = 0;
+            a.items[idx] = w;
+            if (first < 0) first = idx;
+            last = idx;
+            if (!whole) ++n_part;
+            if (!whole && t0 == 0) {
+                // first piece of a split group: the last slice its last slot
+                // reaches is the largest e with sb(e) <= gend
+                const int64_t gend = x - off + wg - 1;
+                int64_t e = ((gend + 1) * v.P - 1) / v.W;
+                if (e > v.P - 1) e = v.P - 1;
+                c.u = u; c.h = w.h; c.qt = w.qt;
+                c.slot0 = w.slot;
+                c.nsplit = (int32_t)(e - b + 1);
             }
         }
         x += len;
     }
+    a.cta_items[2 * b] = (int32_t)(first < 0 ? 0 : first);
+    a.cta_items[2 * b + 1] = (int32_t)(first < 0 ? 0 : last + 1);
 }
-
-// Per-CTA counts packed in one int64 for a single scan: items in bits 0..20,
-// partial pieces in 21..41, combine entries in 42..62 (every total is far
-// below 2^21: items <= groups + CTAs).
-constexpr int PK_SHIFT = 21;
-constexpr int64_t PK_MASK = (1ll << PK_SHIFT) - 1;
 
 constexpr int PLAN_THREADS = 256;
 
@@ -205,89 +227,91 @@ __global__ void __launch_bounds__(PLAN_THREADS) k_plan(ReadoutArgs a)
 {
     pdl_wait();
     ReadoutHeader *hdr = a.header;
-    // [U+1] tb, [U] wg, [grid+1] sb, [grid+1] packed per-CTA counts, [U] nt (int32)
+    // [U+1] tb, [U] wg (int64); [U+1] gb, [U] nt (int32)
     extern __shared__ int64_t s_plan[];
-    int64_t *s_tb = s_plan, *s_wg = s_tb + (a.U + 1), *s_sb = s_wg + a.U, *s_pk = s_sb + (a.grid_ctas + 1);
-    int32_t *s_nt = reinterpret_cast<int32_t *>(s_pk + (a.grid_ctas + 1));
-    for (int u = threadIdx.x; u < a.U; u += blockDim.x) {
-        int cnt = a.count[u];
-        if (cnt < 0 || cnt > a.k_max) {
-            latch_status(a.status, RS3_EINVAL);
-            cnt = cnt < 0 ? 0 : a.k_max;
-        }
-        const int g = a.unit_group[u];
-        if (g < 0 || g >= a.G) {                    // no work for a unit without a valid grid
-            latch_status(a.status, RS3_EINVAL);
-            cnt = 0;
-        }
-        const int64_t *mu = a.meta + (int64_t)u * a.meta_stride_words;
-        const bool sane = mu[BM_HEAD] >= 0 && mu[BM_TAIL] >= mu[BM_HEAD] &&
-                          mu[BM_TAIL] - mu[BM_HEAD] <= a.ring_cap && mu[BM_COND_LEN] >= 0 &&
-                          mu[BM_COND_LEN] <= a.pinned_cap && mu[BM_PTRLEN] >= 0 &&
-                          mu[BM_PTRLEN] <= a.n_ptr;
-        RangeSet rs;
-        if (!sane) {
-            latch_status(a.status, RS3_EINTERNAL);
-            for (int r = 0; r < 4; ++r) { rs.start[r] = 0; rs.len[r] = 0; rs.tiles[r] = 0; }
-            rs.n_tiles = 0; rs.cnt = 0; rs.nq = 0; rs.splits = 1; rs.slot_base = -1;
-        } else {
-            rs = unit_ranges(a, u, cnt);
-        }
-        a.ranges[u] = rs;
-        s_wg[u] = (int64_t)a.plan_ov + rs.n_tiles;
-        s_nt[u] = rs.n_tiles;
-        s_tb[u] = (int64_t)rs.nq * a.H * s_wg[u];   // this unit's slots, scanned below
-    }
-    __syncthreads();
-    // linear slot base of every unit (exclusive scan in rounds of blockDim)
+    int64_t *s_tb = s_plan, *s_wg = s_tb + (a.U + 1);
+    int32_t *s_gb = reinterpret_cast<int32_t *>(s_wg + a.U), *s_nt = s_gb + (a.U + 1);
+    __shared__ int s_np, s_nc;
+    if (threadIdx.x == 0) { s_np = 0; s_nc = 0; }
+    // per unit: the bank's ranges, its groups and their width, scanned into
+    // slot and group bases (rounds of blockDim units)
     int64_t run = 0;
+    int32_t grun = 0;
     for (int u0 = 0; u0 < a.U; u0 += blockDim.x) {
         const int u = u0 + threadIdx.x;
-        const int64_t w = u < a.U ? s_tb[u] : 0;
-        int64_t tot;
-        const int64_t off = block_scan64(w, &tot) + run;
-        if (u < a.U) s_tb[u] = off;
+        int64_t slots = 0;
+        int32_t groups = 0;
+        if (u < a.U) {
+            // every load first (none depends on another), then the checks
+            const int64_t *mu = a.meta + (int64_t)u * a.meta_stride_words;
+            int cnt = a.count[u];
+            const int g = a.unit_group[u];
+            const int64_t head = mu[BM_HEAD], tail = mu[BM_TAIL], cond = mu[BM_COND_LEN], ptr = mu[BM_PTRLEN];
+            if (cnt < 0 || cnt > a.k_max) {
+                latch_status(a.status, RS3_EINVAL);
+                cnt = cnt < 0 ? 0 : a.k_max;
+            }
+            if (g < 0 || g >= a.G) {                // no work for a unit without a valid grid
+                latch_status(a.status, RS3_EINVAL);
+                cnt = 0;
+            }
+            const bool sane = head >= 0 && tail >= head && tail - head <= a.ring_cap && cond >= 0 &&
+                              cond <= a.pinned_cap && ptr >= 0 && ptr <= a.n_ptr;
+            RangeSet rs;
+            if (!sane) {
+                latch_status(a.status, RS3_EINTERNAL);
+                for (int r = 0; r < 4; ++r) { rs.start[r] = 0; rs.len[r] = 0; rs.tiles[r] = 0; }
+                rs.n_tiles = 0; rs.cnt = 0; rs.nq = 0; rs.splits = 1; rs.slot_base = -1;
+            } else {
+                rs = unit_ranges(a, u, cnt);
+            }
+            a.ranges[u] = rs;
+            s_wg[u] = (int64_t)a.plan_ov + rs.n_tiles;
+            s_nt[u] = rs.n_tiles;
+            groups = rs.nq * a.H;
+            slots = (int64_t)groups * s_wg[u];
+        }
+        int64_t off, tot;
+        int32_t goff, gtot;
+        block_scan_pair(slots, groups, off, goff, tot, gtot);
+        if (u < a.U) {
+            s_tb[u] = off + run;
+            s_gb[u] = goff + grun;
+        }
         run += tot;
+        grun += gtot;
     }
-    if (threadIdx.x == 0) s_tb[a.U] = run;
+    if (threadIdx.x == 0) {
+        s_tb[a.U] = run;
+        s_gb[a.U] = grun;
+    }
     int64_t P = (run + a.min_chunk - 1) / a.min_chunk;
     if (P > a.grid_ctas) P = a.grid_ctas;
-    for (int b = threadIdx.x; b <= P; b += blockDim.x) s_sb[b] = P > 0 ? (int64_t)b * run / P : 0;
     __syncthreads();
     PlanView v;
-    v.tb = s_tb; v.wg = s_wg; v.nt = s_nt; v.sb = s_sb; v.U = a.U; v.H = a.H; v.W = run;
+    v.tb = s_tb; v.wg = s_wg; v.nt = s_nt; v.gb = s_gb; v.U = a.U; v.H = a.H; v.W = run;
     v.ov = a.plan_ov;
     v.P = (int)P;
-    // per-CTA counts, then one exclusive scan into offsets
-    for (int b = threadIdx.x; b < v.P; b += blockDim.x) {
-        int ni, np, nc;
-        plan_slice(a, v, b, false, 0, 0, 0, ni, np, nc);
-        s_pk[b] = (int64_t)ni | ((int64_t)np << PK_SHIFT) | ((int64_t)nc << (2 * PK_SHIFT));
+    // every CTA of the launch gets its item range (empty past the P slices);
+    // merge entries are packed through a shared counter
+    for (int b = threadIdx.x; b < a.grid_ctas; b += blockDim.x) {
+        if (b < v.P) {
+            int np;
+            CombineItem c;
+            plan_slice(a, v, b, np, c);
+            if (np) atomicAdd(&s_np, np);
+            if (c.nsplit > 0) a.combine[atomicAdd(&s_nc, 1)] = c;
+        } else {
+            a.cta_items[2 * b] = 0;
+            a.cta_items[2 * b + 1] = 0;
+        }
     }
     __syncthreads();
-    int64_t rsum = 0;
-    for (int b0 = 0; b0 < v.P; b0 += blockDim.x) {
-        const int b = b0 + threadIdx.x;
-        int64_t tot;
-        const int64_t off = block_scan64(b < v.P ? s_pk[b] : 0, &tot) + rsum;
-        if (b < v.P) s_pk[b] = off;
-        rsum += tot;
-    }
-    __syncthreads();
-    for (int b = threadIdx.x; b < v.P; b += blockDim.x) {
-        int ni, np, nc;
-        const int64_t o = s_pk[b];
-        plan_slice(a, v, b, true, o & PK_MASK, (o >> PK_SHIFT) & PK_MASK, (o >> (2 * PK_SHIFT)) & PK_MASK, ni,
-                   np, nc);
-    }
-    const int64_t ri = rsum & PK_MASK, rp = (rsum >> PK_SHIFT) & PK_MASK, rc = (rsum >> (2 * PK_SHIFT)) & PK_MASK;
-    for (int b = threadIdx.x; b <= a.grid_ctas; b += blockDim.x)
-        a.cta_items[b] = (int32_t)(b < v.P ? (s_pk[b] & PK_MASK) : ri);
     if (threadIdx.x == 0) {
-        hdr->n_items = (int32_t)ri;
-        hdr->n_combine = (int32_t)rc;
+        hdr->n_items = (int32_t)(grun + v.P);       // bound on the item indices
+        hdr->n_combine = s_nc;
         hdr->pad[0] = v.P;
-        hdr->pad[1] = (int32_t)rp;                  // partial pieces of all split groups
+        hdr->pad[1] = s_np;                         // partial pieces of all split groups
     }
 }
 
@@ -309,8 +333,8 @@ __global__ void __launch_bounds__(512) k_readout_simt(ReadoutArgs a)
     const int TPR = d / 16;
     float *sK = sm;                      // [SIMT_BN][d]
     float *sV = sm + SIMT_BN * d;        // [SIMT_BN][d]
-    const int it_end = a.cta_items[blockIdx.x + 1];
-    for (int it = a.cta_items[blockIdx.x]; it < it_end; ++it) {
+    const int it_end = a.cta_items[2 * blockIdx.x + 1];
+    for (int it = a.cta_items[2 * blockIdx.x]; it < it_end; ++it) {
         const WorkItem w = a.items[it];
         const RangeSet rs = a.ranges[w.u];
         const int r = threadIdx.x / TPR;
@@ -494,34 +518,41 @@ __global__ void __launch_bounds__(256) k_combine(ReadoutArgs a)
         const int chunk = (int)(task % chunks);
         const int ci = (int)(gr / a.BM), r = (int)(gr % a.BM);
         const CombineItem c = a.combine[ci];
+        if (c.nsplit <= 0) continue;                   // warp-uniform
         const bool whole = !chunked;
         const int j = c.qt * a.BM + r;
         if (j >= a.ranges[c.u].cnt) continue;          // warp-uniform
         int cell = a.idx[(int64_t)c.u * a.k_max + j];
         if (cell < 0 || cell >= a.mn) cell = 0;
-        const float2 *ml = pm + (int64_t)c.slot0 * a.BM + r;      // split s at ml[s * BM]
+        // piece 0 of the group is at slot0; piece s >= 1 is the first item of
+        // slice b0 + s, partial slot 2 (b0 + s).  slot(s) = 2 (b0 + s) + d0 [s = 0]
+        // with d0 = slot0 - 2 b0: a select, no branch, so every piece's loads
+        // can be in flight together
+        const int64_t b0 = c.pad[0], d0 = (int64_t)c.slot0 - 2 * b0;
+        const float2 *ml = pm + 2 * b0 * a.BM + r;                 // piece s at ml[slot_rel(s) BM]
+#define SLOT_REL(s_) (2 * (int64_t)(s_) + ((s_) == 0 ? d0 : 0))
         float M = -INFINITY;
-        for (int s = lane; s < c.nsplit; s += 32) M = fmaxf(M, ml[(int64_t)s * a.BM].x);
+        for (int s = lane; s < c.nsplit; s += 32) M = fmaxf(M, ml[SLOT_REL(s) * a.BM].x);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
         float L = 0.f;
         if (M != -INFINITY)
             for (int s = lane; s < c.nsplit; s += 32) {
-                const float2 v = ml[(int64_t)s * a.BM];
+                const float2 v = ml[SLOT_REL(s) * a.BM];
                 L += exp2f(v.x - M) * v.y;
             }
         L = warp_sum(L);
         const float inv = L > 0.f ? 1.f / L : 0.f;
-        const int64_t sstride = (int64_t)a.BM * d;
+        const int64_t sstride = (int64_t)a.BM * d;                 // one slot
         if (whole) {
             // lanes stride the row's columns four at a time; no warp collectives
             for (int c4 = lane * 4; c4 < d; c4 += 128) {
                 float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-                const float *base = a.part_o + ((int64_t)c.slot0 * a.BM + r) * d + c4;
+                const float *base = a.part_o + (2 * b0 * a.BM + r) * d + c4;
 #pragma unroll 4
                 for (int s = 0; s < c.nsplit; ++s) {
-                    const float ws = M == -INFINITY ? 0.f : exp2f(ml[(int64_t)s * a.BM].x - M);
-                    const float4 po = __ldcs(reinterpret_cast<const float4 *>(base + s * sstride));
+                    const float ws = M == -INFINITY ? 0.f : exp2f(ml[SLOT_REL(s) * a.BM].x - M);
+                    const float4 po = __ldcs(reinterpret_cast<const float4 *>(base + SLOT_REL(s) * sstride));
                     acc.x = fmaf(ws, po.x, acc.x);
                     acc.y = fmaf(ws, po.y, acc.y);
                     acc.z = fmaf(ws, po.z, acc.z);
@@ -534,21 +565,22 @@ __global__ void __launch_bounds__(256) k_combine(ReadoutArgs a)
         }
         const int col = chunk * CW + lane * E;
         if (col >= d) continue;                          // d < 32 only; no collectives below
-        const float *base = a.part_o + ((int64_t)c.slot0 * a.BM + r) * d + col;
+        const float *base = a.part_o + (2 * b0 * a.BM + r) * d + col;
         float acc[E];
 #pragma unroll
         for (int e = 0; e < E; ++e) acc[e] = 0.f;
 #pragma unroll 8
         for (int s = 0; s < c.nsplit; ++s) {
-            const float ws = M == -INFINITY ? 0.f : exp2f(ml[(int64_t)s * a.BM].x - M);
+            const float ws = M == -INFINITY ? 0.f : exp2f(ml[SLOT_REL(s) * a.BM].x - M);
             if constexpr (E == 2) {
-                const float2 po = __ldcs(reinterpret_cast<const float2 *>(base + s * sstride));
+                const float2 po = __ldcs(reinterpret_cast<const float2 *>(base + SLOT_REL(s) * sstride));
                 acc[0] = fmaf(ws, po.x, acc[0]);
                 acc[1] = fmaf(ws, po.y, acc[1]);
             } else {
-                acc[0] = fmaf(ws, __ldcs(base + s * sstride), acc[0]);
+                acc[0] = fmaf(ws, __ldcs(base + SLOT_REL(s) * sstride), acc[0]);
             }
         }
+#undef SLOT_REL
 #pragma unroll
         for (int e = 0; e < E; ++e) acc[e] *= inv;
         store_out_e<T, E>(a, c.u, cell, c.h * d + col, acc);
@@ -562,8 +594,8 @@ __global__ void __launch_bounds__(256) k_combine(ReadoutArgs a)
 // ---------------------------------------------------------------------------
 namespace {
 
-// Bounds of the stream-K plan: items <= groups + CTAs (a slice boundary adds
-// at most one item); a CTA has at most two partial items; at most one combine
+// Bounds of the stream-K plan: item indices < groups + CTAs (group + slice);
+// a CTA has at most two partial items (slots 2b, 2b + 1); at most one merge
 // entry per CTA and per group.
 ReadoutLayout readout_layout(int U, int H, int d, int k_max, int BM, int grid)
 {
@@ -571,13 +603,13 @@ ReadoutLayout readout_layout(int U, int H, int d, int k_max, int BM, int grid)
     const int64_t nq = k_max > 0 ? (k_max + BM - 1) / BM : 1;
     const int64_t groups = (int64_t)U * H * nq;
     L.max_slots = 2 * (int64_t)grid;
-    L.max_combine = groups < grid ? groups : grid;
+    L.max_combine = groups < grid ? groups : grid;   // at most one per CTA slice and per group
     L.max_items = groups + grid;
     size_t off = 0;
     L.header = off;
     off = align_up(off + sizeof(ReadoutHeader), 256);
     L.cta_items = off;
-    off = align_up(off + (size_t)(grid + 1) * 4, 256);
+    off = align_up(off + (size_t)grid * 2 * 4, 256);   // [begin, end) per CTA
     L.ranges = off;
     off = align_up(off + (size_t)U * sizeof(RangeSet), 256);
     L.items = off;
@@ -647,8 +679,8 @@ rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, in
         return RS3_EINVAL;
     const ReadoutPath p = choose_readout_path(dtype, d);
     const ReadoutLayout L = readout_layout(bank->U, H, d, k_max, p.BM, p.grid);
-    // the plan packs its per-CTA counts into PK_SHIFT-bit fields
-    if (L.max_items >= PK_MASK || L.max_slots >= PK_MASK || L.max_combine >= PK_MASK) return RS3_EUNSUPPORTED;
+    // work-item indices (group + slice) and item ranges are 32-bit
+    if (L.max_items >= ((int64_t)1 << 30) || L.max_slots >= ((int64_t)1 << 30)) return RS3_EUNSUPPORTED;
     if (workspace_bytes < L.total) return RS3_ECAPACITY;
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     a->q = q;
@@ -714,8 +746,8 @@ rs3_status launch_attend(const ReadoutArgs &a, const ReadoutPath &p, rs3_dtype d
                    static_cast<const uint4 *>(a.residual), static_cast<uint4 *>(a.out), nvec);
         if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     }
-    // plan shared memory: unit slot bases and widths, slice bounds, per-CTA counts, unit tiles
-    const size_t plan_smem = ((size_t)(2 * a.U + 1) + 2 * (size_t)(a.grid_ctas + 1)) * 8 + (size_t)a.U * 4;
+    // plan shared memory: unit slot bases and widths (int64), group bases and tiles (int32)
+    const size_t plan_smem = (size_t)(2 * a.U + 1) * 8 + (size_t)(2 * a.U + 1) * 4;
     if (rs3_kernel_smem((const void *)k_plan, plan_smem) != RS3_OK) return RS3_EUNSUPPORTED;
     launch_pdl(k_plan, dim3(1), dim3(PLAN_THREADS), plan_smem, st, a);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;

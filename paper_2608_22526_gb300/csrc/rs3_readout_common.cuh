@@ -27,7 +27,7 @@ struct ReadoutArgs {
     int64_t max_slots;
     int64_t max_items;
     int grid_ctas;          // CTAs of the readout launch (the plan's slice count bound)
-    int32_t *cta_items;     // [grid_ctas + 1]: CTA b runs items [cta_items[b], cta_items[b+1])
+    int32_t *cta_items;     // [grid_ctas][2]: CTA b runs items [cta_items[2b], cta_items[2b+1])
     float scale_log2;       // softmax scale * log2(e)
     uint64_t wait_ns;       // limit of each device-side wait (global-timer ns)
     ReadoutHeader *header;

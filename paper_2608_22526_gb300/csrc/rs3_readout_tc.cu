@@ -219,7 +219,7 @@ k_readout_tc(const ReadoutArgs a, const __grid_constant__ CUtensorMap tmk,
     // previous kernel of the stream has completed
     pdl_wait();
     // this CTA's slice of the stream-K plan
-    const int it_begin = a.cta_items[blockIdx.x], it_end = a.cta_items[blockIdx.x + 1];
+    const int it_begin = a.cta_items[2 * blockIdx.x], it_end = a.cta_items[2 * blockIdx.x + 1];
 
     if ((warp == 0 || warp == 2) && lane == 0) {
         // ------------------------------------------------------------------

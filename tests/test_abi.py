@@ -138,17 +138,17 @@ def test_mask_calls_reject_bad_arguments_on_host(binding):
 
 
 def test_oversized_readout_plan_is_refused(binding):
-    """The readout's work list packs per-CTA counts into 21-bit fields: a
-    request whose list could reach 2^21 entries (4096 units, k_max 16384 on
-    the fp32 path: 4096 x 512 query tiles) is refused on the host with
-    RS3_EUNSUPPORTED; a small request with the same descriptor shape gets as
-    far as the workspace-size check."""
+    """The readout's work-item indices are 32-bit: a request whose list could
+    reach 2^30 entries (4096 units x 512 heads x 512 query tiles of the fp32
+    path, k_max 16384) is refused on the host with RS3_EUNSUPPORTED; a small
+    request with the same descriptor shape gets as far as the workspace-size
+    check."""
     lib = binding.lib
     one = ctypes.c_void_p(16)
 
     def bank(U):
         b = binding.BankDesc()
-        b.U, b.H, b.d, b.D, b.dtype, b.mn = U, 1, 64, 64, 0, 16384
+        b.U, b.H, b.d, b.D, b.dtype, b.mn = U, 512, 16, 512 * 16, 0, 16384
         b.n_cond, b.window, b.max_frames, b.n_ptr = 0, -1, 4, 0
         b.pinned_cap, b.ring_cap, b.rows_per_unit, b.meta_stride = 0, 64, 64, 8 * 24
         b.k_store = b.v_store = b.meta = one
@@ -156,7 +156,7 @@ def test_oversized_readout_plan_is_refused(binding):
         return b
 
     big, small = bank(4096), bank(8)
-    args = lambda b, ws: (one, 0, 1, 16384, 1, 64, one, one, one, 16384, ctypes.byref(b), None, None,
+    args = lambda b, ws: (one, 0, 1, 16384, 512, 16, one, one, one, 16384, ctypes.byref(b), None, None,
                           one, 0.0, one, ws, one, None)
     assert lib.rs3_memory_readout(*args(big, 1 << 62)) == binding.RS3_EUNSUPPORTED
     assert lib.rs3_memory_readout_attend(*args(big, 1 << 62)) == binding.RS3_EUNSUPPORTED
