@@ -139,6 +139,7 @@ struct PlanView {
     const int64_t *wg;   // [U]   slots per group of each unit
     const int32_t *nt;   // [U]   key tiles of each unit
     const int32_t *gb;   // [U+1] first linear group of each unit
+    const int32_t *cnt;  // [U]   kept queries of each unit
     int U, H;
     int64_t W;
     int P;
@@ -178,7 +179,7 @@ __device__ void plan_slice(const ReadoutArgs &a, const PlanView &v, int b, int &
     int64_t first = -1, last = -1;
     c.u = c.h = c.qt = c.slot0 = c.nsplit = 0;
     c.pad[0] = b;
-    c.pad[1] = c.pad[2] = 0;
+    c.pad[1] = c.pad[2] = 0;                      // pad[1]: the unit's kept queries
     n_part = 0;
     for (int64_t x = lo; x < hi;) {
         int u, gl;
@@ -213,6 +214,7 @@ __device__ void plan_slice(const ReadoutArgs &a, const PlanView &v, int b, int &
                 c.u = u; c.h = w.h; c.qt = w.qt;
                 c.slot0 = w.slot;
                 c.nsplit = (int32_t)(e - b + 1);
+                c.pad[1] = v.cnt[u];
             }
         }
         x += len;
@@ -230,7 +232,7 @@ __global__ void __launch_bounds__(PLAN_THREADS) k_plan(ReadoutArgs a)
     // [U+1] tb, [U] wg (int64); [U+1] gb, [U] nt (int32)
     extern __shared__ int64_t s_plan[];
     int64_t *s_tb = s_plan, *s_wg = s_tb + (a.U + 1);
-    int32_t *s_gb = reinterpret_cast<int32_t *>(s_wg + a.U), *s_nt = s_gb + (a.U + 1);
+    int32_t *s_gb = reinterpret_cast<int32_t *>(s_wg + a.U), *s_nt = s_gb + (a.U + 1), *s_cnt = s_nt + a.U;
     __shared__ int s_np, s_nc;
     if (threadIdx.x == 0) { s_np = 0; s_nc = 0; }
     // per unit: the bank's ranges, its groups and their width, scanned into
@@ -268,6 +270,7 @@ __global__ void __launch_bounds__(PLAN_THREADS) k_plan(ReadoutArgs a)
             a.ranges[u] = rs;
             s_wg[u] = (int64_t)a.plan_ov + rs.n_tiles;
             s_nt[u] = rs.n_tiles;
+            s_cnt[u] = rs.cnt;
             groups = rs.nq * a.H;
             slots = (int64_t)groups * s_wg[u];
         }
@@ -289,7 +292,7 @@ __global__ void __launch_bounds__(PLAN_THREADS) k_plan(ReadoutArgs a)
     if (P > a.grid_ctas) P = a.grid_ctas;
     __syncthreads();
     PlanView v;
-    v.tb = s_tb; v.wg = s_wg; v.nt = s_nt; v.gb = s_gb; v.U = a.U; v.H = a.H; v.W = run;
+    v.tb = s_tb; v.wg = s_wg; v.nt = s_nt; v.gb = s_gb; v.cnt = s_cnt; v.U = a.U; v.H = a.H; v.W = run;
     v.ov = a.plan_ov;
     v.P = (int)P;
     // every CTA of the launch gets its item range (empty past the P slices);
@@ -519,18 +522,82 @@ __global__ void __launch_bounds__(256) k_combine(ReadoutArgs a)
         const int ci = (int)(gr / a.BM), r = (int)(gr % a.BM);
         const CombineItem c = a.combine[ci];
         if (c.nsplit <= 0) continue;                   // warp-uniform
-        const bool whole = !chunked;
         const int j = c.qt * a.BM + r;
-        if (j >= a.ranges[c.u].cnt) continue;          // warp-uniform
-        int cell = a.idx[(int64_t)c.u * a.k_max + j];
-        if (cell < 0 || cell >= a.mn) cell = 0;
+        if (j >= c.pad[1]) continue;                   // the unit's kept queries (warp-uniform)
         // piece 0 of the group is at slot0; piece s >= 1 is the first item of
         // slice b0 + s, partial slot 2 (b0 + s).  slot(s) = 2 (b0 + s) + d0 [s = 0]
         // with d0 = slot0 - 2 b0: a select, no branch, so every piece's loads
         // can be in flight together
         const int64_t b0 = c.pad[0], d0 = (int64_t)c.slot0 - 2 * b0;
         const float2 *ml = pm + 2 * b0 * a.BM + r;                 // piece s at ml[slot_rel(s) BM]
+        const int64_t sstride = (int64_t)a.BM * d;                 // one slot
 #define SLOT_REL(s_) (2 * (int64_t)(s_) + ((s_) == 0 ? d0 : 0))
+        if (!chunked) {
+            // One round trip for the row's cell, the pieces' (m, l) pairs (lane
+            // s holds piece s) and the first MP pieces' partial columns (lanes
+            // stride the row four columns at a time); the weights follow.
+            constexpr int MP = 4;
+            int cell = a.idx[(int64_t)c.u * a.k_max + j];
+            const float2 mv = lane < c.nsplit ? ml[SLOT_REL(lane) * a.BM] : make_float2(-INFINITY, 0.f);
+            const float *base = a.part_o + (2 * b0 * a.BM + r) * d;
+            float4 pf[MP][2];
+#pragma unroll
+            for (int q = 0; q < MP; ++q)
+#pragma unroll
+                for (int cb = 0; cb < 2; ++cb) {
+                    const int c4 = lane * 4 + 128 * cb;
+                    pf[q][cb] = (q < c.nsplit && c4 < d)
+                                    ? __ldcs(reinterpret_cast<const float4 *>(base + SLOT_REL(q) * sstride + c4))
+                                    : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+            float M = mv.x;
+            for (int s = lane + 32; s < c.nsplit; s += 32) M = fmaxf(M, ml[SLOT_REL(s) * a.BM].x);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+            float L = 0.f;
+            if (M != -INFINITY) {
+                if (lane < c.nsplit) L = exp2f(mv.x - M) * mv.y;
+                for (int s = lane + 32; s < c.nsplit; s += 32) {
+                    const float2 v = ml[SLOT_REL(s) * a.BM];
+                    L += exp2f(v.x - M) * v.y;
+                }
+            }
+            L = warp_sum(L);
+            const float inv = L > 0.f ? 1.f / L : 0.f;
+            float wq[MP];
+#pragma unroll
+            for (int q = 0; q < MP; ++q) {
+                const float mq = __shfl_sync(0xffffffffu, mv.x, q);
+                wq[q] = (q < c.nsplit && M != -INFINITY) ? exp2f(mq - M) : 0.f;
+            }
+            if (cell < 0 || cell >= a.mn) cell = 0;
+#pragma unroll
+            for (int cb = 0; cb < 2; ++cb) {
+                const int c4 = lane * 4 + 128 * cb;
+                if (c4 >= d) continue;
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int q = 0; q < MP; ++q) {
+                    acc.x = fmaf(wq[q], pf[q][cb].x, acc.x);
+                    acc.y = fmaf(wq[q], pf[q][cb].y, acc.y);
+                    acc.z = fmaf(wq[q], pf[q][cb].z, acc.z);
+                    acc.w = fmaf(wq[q], pf[q][cb].w, acc.w);
+                }
+                for (int s = MP; s < c.nsplit; ++s) {
+                    const float ws = M == -INFINITY ? 0.f : exp2f(ml[SLOT_REL(s) * a.BM].x - M);
+                    const float4 po = __ldcs(reinterpret_cast<const float4 *>(base + SLOT_REL(s) * sstride + c4));
+                    acc.x = fmaf(ws, po.x, acc.x);
+                    acc.y = fmaf(ws, po.y, acc.y);
+                    acc.z = fmaf(ws, po.z, acc.z);
+                    acc.w = fmaf(ws, po.w, acc.w);
+                }
+                const float o4[4] = {acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv};
+                store_out4<T>(a, c.u, cell, c.h * d + c4, o4);
+            }
+            continue;
+        }
+        int cell = a.idx[(int64_t)c.u * a.k_max + j];
+        if (cell < 0 || cell >= a.mn) cell = 0;
         float M = -INFINITY;
         for (int s = lane; s < c.nsplit; s += 32) M = fmaxf(M, ml[SLOT_REL(s) * a.BM].x);
 #pragma unroll
@@ -543,26 +610,6 @@ __global__ void __launch_bounds__(256) k_combine(ReadoutArgs a)
             }
         L = warp_sum(L);
         const float inv = L > 0.f ? 1.f / L : 0.f;
-        const int64_t sstride = (int64_t)a.BM * d;                 // one slot
-        if (whole) {
-            // lanes stride the row's columns four at a time; no warp collectives
-            for (int c4 = lane * 4; c4 < d; c4 += 128) {
-                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-                const float *base = a.part_o + (2 * b0 * a.BM + r) * d + c4;
-#pragma unroll 4
-                for (int s = 0; s < c.nsplit; ++s) {
-                    const float ws = M == -INFINITY ? 0.f : exp2f(ml[SLOT_REL(s) * a.BM].x - M);
-                    const float4 po = __ldcs(reinterpret_cast<const float4 *>(base + SLOT_REL(s) * sstride));
-                    acc.x = fmaf(ws, po.x, acc.x);
-                    acc.y = fmaf(ws, po.y, acc.y);
-                    acc.z = fmaf(ws, po.z, acc.z);
-                    acc.w = fmaf(ws, po.w, acc.w);
-                }
-                const float o4[4] = {acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv};
-                store_out4<T>(a, c.u, cell, c.h * d + c4, o4);
-            }
-            continue;
-        }
         const int col = chunk * CW + lane * E;
         if (col >= d) continue;                          // d < 32 only; no collectives below
         const float *base = a.part_o + (2 * b0 * a.BM + r) * d + col;
@@ -746,8 +793,8 @@ rs3_status launch_attend(const ReadoutArgs &a, const ReadoutPath &p, rs3_dtype d
                    static_cast<const uint4 *>(a.residual), static_cast<uint4 *>(a.out), nvec);
         if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     }
-    // plan shared memory: unit slot bases and widths (int64), group bases and tiles (int32)
-    const size_t plan_smem = (size_t)(2 * a.U + 1) * 8 + (size_t)(2 * a.U + 1) * 4;
+    // plan shared memory: unit slot bases and widths (int64), group bases, tiles, kept queries (int32)
+    const size_t plan_smem = (size_t)(2 * a.U + 1) * 8 + (size_t)(3 * a.U + 1) * 4;
     if (rs3_kernel_smem((const void *)k_plan, plan_smem) != RS3_OK) return RS3_EUNSUPPORTED;
     launch_pdl(k_plan, dim3(1), dim3(PLAN_THREADS), plan_smem, st, a);
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
