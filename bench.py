@@ -191,6 +191,7 @@ class DeviceSequence:
         self.masks_np = masks
         self.T = T
         self.P = w.prefill_frames
+        self.rope = None        # RoPE table [mn][d/2][2] when queries and keys are rotated (Eq. 7)
 
     def frame(self, key, t):
         """Device tensor of input `key` for frame t."""
@@ -281,13 +282,14 @@ def run_step(pipe, data, timers=None, side=None, merge=None, att_ev=None):
         if timers is not None:
             sel_t[t][1] = ev
 
+    rope = getattr(data, "rope", None)
     first = data.P + (1 if w.n_cond > 0 else 0)
     for t in range(data.T):
         if t < data.P:                       # unpruned frames already in the bank
-            pipe.commit(F("k", t), F("v", t), None, 0)
+            pipe.commit(F("k", t), F("v", t), None, 0, rope=rope)
             continue
         if t == data.P and w.n_cond > 0:
-            pipe.commit(F("k", t), F("v", t), F("mask", t), 1)
+            pipe.commit(F("k", t), F("v", t), F("mask", t), 1, rope=rope)
             if data.ptr is not None:
                 pipe.set_pointers(*data.ptr)
             continue
@@ -303,19 +305,19 @@ def run_step(pipe, data, timers=None, side=None, merge=None, att_ev=None):
             e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
             e[0].record(main)
         if mrg is main:
-            pipe.readout(F("z", t), F("x", t), F("x", t))        # both phases, one call
+            pipe.readout(F("z", t), F("x", t), F("x", t), rope=rope)   # both phases, one call
         else:
             if att_ev is not None:
                 ea = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
                 ea[0].record(main)
-            pipe.readout_attend(F("z", t), F("x", t), F("x", t))
+            pipe.readout_attend(F("z", t), F("x", t), F("x", t), rope=rope)
             if att_ev is not None:
                 ea[1].record(main)
                 att_ev.append(ea)
             att = torch.cuda.Event()
             att.record(main)
             mrg.wait_event(att)
-            pipe.readout_merge(F("z", t), F("x", t), F("x", t), stream=mrg)
+            pipe.readout_merge(F("z", t), F("x", t), F("x", t), rope=rope, stream=mrg)
         ev = torch.cuda.Event(enable_timing=timers is not None)
         ev.record(mrg)
         rd_ev[t] = ev                        # frame t's keep-set and workspace are free
@@ -324,7 +326,7 @@ def run_step(pipe, data, timers=None, side=None, merge=None, att_ev=None):
         if timers is not None:
             e[1] = ev
             e[2].record(main)
-        pipe.commit(F("k", t), F("v", t), F("mask", t), 0)
+        pipe.commit(F("k", t), F("v", t), F("mask", t), 0, rope=rope)
         if timers is not None:
             e[3].record(main)
             timers.append((t, [sel_t[t][0], sel_t[t][1], e[0], e[1], e[2], e[3]]))
@@ -405,16 +407,19 @@ def gpu_arm(args):
     w = synth.WORKLOADS[args.workload]
     hbm, tc_burst, tc_sust, peak_src = _peaks()
 
-    def build(dense):
+    def build(dense, rope=False):
         data = DeviceSequence(w, dense, device)
+        if rope:                                    # Eq. 7: queries and keys rotated by their own cell
+            data.rope = torch.from_numpy(synth.Sequence(w).rope_table()).to(device)
         pipe = Pipeline(w, device=device, dense=dense)
         torch.cuda.synchronize()        # inputs and bank set-up ran on the default stream
         return pipe, data
 
     results = {}
     reps = None
-    for mode in (["pruned", "dense"] if not args.no_dense else ["pruned"]):
-        pipe, data = build(mode == "dense")
+    modes = ["pruned"] + ([] if args.no_dense else ["dense"]) + ([] if args.no_rope else ["rope"])
+    for mode in modes:
+        pipe, data = build(mode == "dense", rope=mode == "rope")
         stream = torch.cuda.Stream()
         side = torch.cuda.Stream()      # selection of frame t+1 runs beside frame t
         merge = torch.cuda.Stream()     # split-KV merge of frame t beside its commit
@@ -604,6 +609,17 @@ def gpu_arm(args):
     line["commit_frac_hbm"] = round(line["commit_gbs"] / hbm, 4)
     line["per_call_note"] = ("select_ms, readout_call_ms and commit_ms are CUDA-event times of each "
                              "call issued on its own outside the graph (host launch included)")
+    if "rope" in results:
+        Rn = results["rope"]
+        rope_fps = frames_per_pass * reps * args.steps / Rn["dev_s"]
+        line["rope"] = {"value": round(rope_fps, 2), "unit": "frames/s",
+                        "what": "Eq. 7 on: each kept query rotated by its own cell in the readout's query "
+                                "load, each key stored rotated by its own cell at commit (SAM2-style 2-D "
+                                "axial table; pointer rows unrotated)",
+                        "cost_vs_off": round(1.0 - rope_fps / value, 4) if world == 1 else None}
+        if Rn["att_ms"] and P["att_ms"]:
+            line["rope"]["attend_us"] = round(1e3 * float(np.mean(Rn["att_ms"])), 3)
+            line["rope"]["attend_us_off"] = round(1e3 * float(np.mean(P["att_ms"])), 3)
     if "dense" in results:
         Dn = results["dense"]
         dense_fps = frames_per_pass * reps * args.steps / Dn["dev_s"]
@@ -618,6 +634,8 @@ def gpu_arm(args):
                        "note": "a step here is one pass of the sequence with its copies"}
     if not args.no_decoder:
         line["close_argmax"] = measure_close_argmax(w, device, hbm)
+    if args.growth_frames > 0 and world == 1:
+        line["bank_growth"] = bank_growth(device, args.growth_frames)
     if not args.no_cpu_baseline and world == 1:
         line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_seconds)
     print(json.dumps(line), flush=True)
@@ -648,6 +666,70 @@ def bank_summary(w, lens, dense_lens=None):
         dp = max(sum(n) for n in dense_lens)
         out.update({"dense_peak_rows": int(dp), "dense_peak_bytes": int(dp * 2 * w.D * b),
                     "reduction": round(1.0 - peak / dp, 4) if dp else None})
+    return out
+
+
+GROWTH_DW = (12, 24)
+
+
+def bank_growth(device, frames: int):
+    """Bank growth under the paper's write keep-set (Sec. 3.2, Eq. 8) on the
+    first `frames` frames of the long-video stream: K_w = the object's first
+    mask dilated by D_w grid cells (with the 5% / 95% fall-through), computed
+    on the device and held fixed, so every frame adds |K_w| rows.  Each D_w
+    runs the whole sequence (selection, readout over the growing bank, commit
+    of K_w) as one CUDA graph: frames/s over two timed passes, and the bank
+    rows / K + V bytes it ends with against the unpruned bank (every cell of
+    every frame) and the per-frame masks the benchmark workloads commit."""
+    import torch
+    from paper_2608_22526_gb300 import rs3, synth
+    from paper_2608_22526_gb300.pipeline import Pipeline
+    w = synth.scaled(synth.WORKLOADS["long_video"], frames=frames, name_suffix="")
+    seq = synth.Sequence(w)
+    b = 2 if w.dtype == "bf16" else 4
+    row_bytes = 2 * w.D * b
+    masks_rows = int(sum(int(seq.masks(t).astype(np.int64).sum()) for t in range(w.frames)))
+    out = {"workload": f"long_video, first {w.frames} frames (64x64 grid, 1x256 heads, unbounded bank)",
+           "frames": w.frames,
+           "unpruned": {"rows": w.frames * w.mn * w.U, "bytes": w.frames * w.mn * w.U * row_bytes},
+           "per_frame_masks": {"rows": masks_rows, "bytes": masks_rows * row_bytes},
+           "paper_kw": []}
+    ug = torch.tensor(w.unit_group(), dtype=torch.int32, device=device)
+    data = DeviceSequence(w, False, device)          # the inputs once; only the commit mask changes
+    for dw in GROWTH_DW:
+        p = rs3.default_params(rho=w.rho, r_s=w.r_s, c=w.c, union_mode=w.union_mode, D_w=dw)
+        seed = torch.from_numpy(np.ascontiguousarray(seq.masks(0))).to(device)
+        kw = torch.empty((w.U, w.mn), dtype=torch.uint8, device=device)
+        st = torch.zeros(1, dtype=torch.int32, device=device)
+        rs3.rs3_write_keepset(seed, ug, w.U, w.m, w.n, p, kw, st)
+        n_kw = int(kw.to(torch.int64).sum().item())
+        data.dev["mask"][:] = kw                     # every frame commits the fixed K_w
+        pipe = Pipeline(w, device=device, ring_cap=w.frames * w.mn, params=p)
+        torch.cuda.synchronize()
+        stream, side, merge = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+        with torch.cuda.stream(stream):
+            run_step(pipe, data, side=side, merge=merge)
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                run_step(pipe, data, side=side, merge=merge)
+            g.replay()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(2):
+                g.replay()
+            e1.record(stream)
+            torch.cuda.synchronize()
+        secs = e0.elapsed_time(e1) / 1e3 / 2
+        meta, _ = rs3.rs3_bank_read_meta(pipe.bank)
+        rows = int(meta[:, 7].sum())
+        assert int(pipe.status.item()) == 0 and rows == w.frames * n_kw, "bank stride differs from |K_w|"
+        out["paper_kw"].append({"D_w": dw, "kw_rows_per_frame": n_kw, "rows": rows, "bytes": rows * row_bytes,
+                                "reduction_vs_unpruned": round(1.0 - rows / out["unpruned"]["rows"], 4),
+                                "frames_per_s": round((w.frames - 1) / secs, 2)})
+        del pipe, g
+        torch.cuda.empty_cache()
     return out
 
 
@@ -859,8 +941,11 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--no-dense", action="store_true")
+    ap.add_argument("--no-rope", action="store_true", help="skip the RoPE-on (queries and keys) pass")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-decoder", action="store_true", help="skip the decoder-side kernel measurement")
+    ap.add_argument("--growth-frames", type=int, default=300,
+                    help="frames of the long-video bank-growth study under the paper's write keep-set (0: skip)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--reps", type=int, default=0, help="sequence passes per step (0: about 50 ms)")

@@ -246,6 +246,25 @@ rs3_status rs3_bank_commit(const rs3_bank *bank, const void *k_new, const void *
                            const uint8_t *keep_mask, int is_cond, int32_t *status,
                            rs3_stream_t stream);
 
+/* rs3_bank_commit with RoPE on the key side (Sec. 3.1, Eq. 7: keys are
+ * rotated by their own grid position, as the queries are by theirs).  Every
+ * kept key row k_new[u][i] is stored rotated by the (cos, sin) of its own
+ * cell i: in each head, elements (2p, 2p+1) become
+ *   (k0 cos - k1 sin, k0 sin + k1 cos),  (cos, sin) = rope_cos_sin[i][p]
+ * computed in fp32 and rounded once to the bank dtype (nearest-even for
+ * bf16).  Values are stored as given.  A rotation is linear in the key and
+ * depends only on the key's own cell, so storing rotated keys and rotating
+ * them at every read give the same attention; the commit does it once per
+ * key.  Pointer rows (rs3_bank_set_pointers) are stored unrotated: object
+ * pointers carry no grid position.
+ * rope_cos_sin: device fp32 [mn][d/2][2], the same table rs3_memory_readout
+ * takes for the queries, 16-byte aligned.  Errors as rs3_bank_commit, plus
+ * RS3_EINVAL for a NULL or misaligned table and RS3_EUNSUPPORTED when d is
+ * not a multiple of 8. */
+rs3_status rs3_bank_commit_rope(const rs3_bank *bank, const void *k_new, const void *v_new,
+                                const uint8_t *keep_mask, int is_cond, const float *rope_cos_sin,
+                                int32_t *status, rs3_stream_t stream);
+
 /* Replaces every unit's pointer rows with k_ptr[u], v_ptr[u] (device
  * [U][n_ptr][D]).  RS3_EINVAL when the bank has n_ptr == 0. */
 rs3_status rs3_bank_set_pointers(const rs3_bank *bank, const void *k_ptr, const void *v_ptr,

@@ -12,6 +12,7 @@ memory bank.  Each function cites the part of the paper it follows:
   readout()        Sec. 3.1: Eq. 6 sparse memory attention, Eq. 7 RoPE gather
   scatter_output() Sec. 3.1: Eq. 6 scatter S_K back onto the m x n grid
   OracleBank       Sec. 3.2: Eq. 8 write-pruned commit, Algorithm 1 sparse write
+  rotate_rows()    Sec. 3.1: Eq. 7 on the key side (keys rotated by their own cell)
   write_keepset()  Sec. 3.2: Eq. 8 with the 5% / 95% fall-through
   close_argmax()   Sec. 3.3: 9 x 9 closure per object, then the palette argmax
   downsample(), seed_track()
@@ -241,6 +242,21 @@ def scatter_output(residual: Optional[np.ndarray], dtype: str, mn: int, D: int,
 # write side (Sec. 3.2)
 # ---------------------------------------------------------------------------
 
+def rotate_rows(x: np.ndarray, dtype: str, rope: np.ndarray) -> np.ndarray:
+    """Eq. 7 applied to the keys: row i of x [mn, H*d] (stored dtype) rotated
+    by the table entries of its own cell i -- in every head, elements
+    (2p, 2p+1) turn by the angle whose (cos, sin) is rope[i, p] -- in fp64,
+    then rounded once to the stored dtype.  rope: [mn, d/2, 2]."""
+    rope = np.asarray(rope, dtype=np.float64)
+    mn, half = rope.shape[0], rope.shape[1]
+    xd = widen(x, dtype).astype(np.float64).reshape(mn, -1, half, 2)      # [mn, H, d/2, (even, odd)]
+    cs = rope[:, None, :, 0]
+    sn = rope[:, None, :, 1]
+    ev, od = xd[..., 0], xd[..., 1]
+    y = np.stack([ev * cs - od * sn, ev * sn + od * cs], axis=-1)
+    return round_to(y.reshape(mn, -1), dtype)
+
+
 def write_keepset(seeds: np.ndarray, unit_group: np.ndarray, m: int, n: int, D_w: int,
                   fall_lo: float = 0.05, fall_hi: float = 0.95, fall_through: int = 1,
                   union_mode: int = 1) -> np.ndarray:
@@ -283,9 +299,13 @@ class OracleBank:
             self.ptr_len[u] = 0
 
     def commit(self, knew: np.ndarray, vnew: np.ndarray, mask: Optional[np.ndarray],
-               is_cond: int) -> List[int]:
+               is_cond: int, rope: Optional[np.ndarray] = None) -> List[int]:
         """Algorithm 1's sparse write for every unit: rows with mask = 1, in
-        ascending grid order.  Returns the per-unit status (0 or 2 = capacity)."""
+        ascending grid order.  With a RoPE table every key row is first rotated
+        by its own cell (rotate_rows), so the bank holds rotated keys.  Returns
+        the per-unit status (0 or 2 = capacity)."""
+        if rope is not None:
+            knew = np.stack([rotate_rows(knew[u], self.dtype, rope) for u in range(self.U)])
         st = []
         row_bytes = self.D * np.dtype(self.npdt).itemsize
         for u in range(self.U):

@@ -46,6 +46,34 @@ __device__ __forceinline__ void copy_row(uint4 *__restrict__ dk, uint4 *__restri
     }
 }
 
+// Eq. 7 on the key side: one 16-byte piece of a key row (bf16: four pairs,
+// fp32: two pairs; element 2i and 2i + 1 of a head form pair i) rotated by
+// the (cos, sin) of those pairs at the row's own cell, in fp32, then rounded
+// once to the stored type.  f points at the first pair's (cos, sin).
+__device__ __forceinline__ uint4 rotate_piece(uint4 v, const float *__restrict__ f, int esz)
+{
+    if (esz == 2) {
+        const float4 a = __ldg(reinterpret_cast<const float4 *>(f));
+        const float4 b = __ldg(reinterpret_cast<const float4 *>(f) + 1);
+        const float cs[4] = {a.x, a.z, b.x, b.z}, sn[4] = {a.y, a.w, b.y, b.w};
+        uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float x0 = __uint_as_float(w[i] << 16), x1 = __uint_as_float(w[i] & 0xffff0000u);
+            const float y0 = x0 * cs[i] - x1 * sn[i], y1 = x0 * sn[i] + x1 * cs[i];
+            uint32_t r;
+            asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(y1), "f"(y0));
+            w[i] = r;
+        }
+        return make_uint4(w[0], w[1], w[2], w[3]);
+    }
+    const float4 a = __ldg(reinterpret_cast<const float4 *>(f));
+    const float x0 = __uint_as_float(v.x), x1 = __uint_as_float(v.y);
+    const float x2 = __uint_as_float(v.z), x3 = __uint_as_float(v.w);
+    return make_uint4(__float_as_uint(x0 * a.x - x1 * a.y), __float_as_uint(x0 * a.y + x1 * a.x),
+                      __float_as_uint(x2 * a.z - x3 * a.w), __float_as_uint(x2 * a.w + x3 * a.z));
+}
+
 // Number of nonzero bytes in a 16-byte word.
 __device__ __forceinline__ int nonzero_bytes(uint4 w)
 {
@@ -64,7 +92,8 @@ __device__ __forceinline__ int nonzero_bytes(uint4 w)
 __global__ void __launch_bounds__(256)
 k_commit(const uint8_t *__restrict__ k_new, const uint8_t *__restrict__ v_new,
          const uint8_t *__restrict__ mask, int mn, int is_cond, int64_t row_bytes, BankDev bk,
-         uint8_t *__restrict__ k_store, uint8_t *__restrict__ v_store, int32_t *status)
+         uint8_t *__restrict__ k_store, uint8_t *__restrict__ v_store, int32_t *status,
+         const float *__restrict__ rope, int d, int esz)
 {
     pdl_wait();
     __shared__ int32_t s_list[COMMIT_CHUNK];
@@ -165,6 +194,7 @@ k_commit(const uint8_t *__restrict__ k_new, const uint8_t *__restrict__ v_new,
         for (int i0 = threadIdx.x; i0 < npiece; i0 += 4 * blockDim.x) {
             uint4 kk[4], vv[4];
             int64_t dst[4];
+            int cellq[4], eq[4];
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int i = i0 + q * blockDim.x;
@@ -172,6 +202,8 @@ k_commit(const uint8_t *__restrict__ k_new, const uint8_t *__restrict__ v_new,
                     const int j = i / nvec, v = i - j * nvec;
                     const int64_t so = (int64_t)s_list[j] * row_bytes + 16 * v;
                     dst[q] = s_row[j] * row_bytes + 16 * v;
+                    cellq[q] = s_list[j];
+                    eq[q] = (16 * v) / esz;                  // first element of the piece
                     kk[q] = __ldcs(reinterpret_cast<const uint4 *>(ksrc + so));
                     vv[q] = __ldcs(reinterpret_cast<const uint4 *>(vsrc + so));
                 }
@@ -179,6 +211,9 @@ k_commit(const uint8_t *__restrict__ k_new, const uint8_t *__restrict__ v_new,
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 if (i0 + q * (int)blockDim.x < npiece) {
+                    if (rope)                              // keys stored rotated by their own cell
+                        kk[q] = rotate_piece(kk[q], rope + ((int64_t)cellq[q] * (d / 2) + (eq[q] % d) / 2) * 2,
+                                             esz);
                     *reinterpret_cast<uint4 *>(kdst + dst[q]) = kk[q];
                     *reinterpret_cast<uint4 *>(vdst + dst[q]) = vv[q];
                 }
@@ -309,9 +344,10 @@ extern "C" rs3_status rs3_bank_init(rs3_bank *bank, int U, int H, int d, rs3_dty
     return RS3_OK;
 }
 
-extern "C" rs3_status rs3_bank_commit(const rs3_bank *bank, const void *k_new, const void *v_new,
-                                      const uint8_t *keep_mask, int is_cond, int32_t *status,
-                                      rs3_stream_t stream)
+namespace {
+
+rs3_status commit_launch(const rs3_bank *bank, const void *k_new, const void *v_new, const uint8_t *keep_mask,
+                         int is_cond, const float *rope, int32_t *status, rs3_stream_t stream)
 {
     if (!bank_ok(bank) || !k_new || !v_new || !status) return RS3_EINVAL;
     if (is_cond != 0 && is_cond != 1) return RS3_EINVAL;
@@ -324,9 +360,28 @@ extern "C" rs3_status rs3_bank_commit(const rs3_bank *bank, const void *k_new, c
     const int64_t row_bytes = (int64_t)bank->D * (int64_t)elem_bytes(bank->dtype);
     launch_pdl(k_commit, dim3(nchunks, bank->U), dim3(256), 0, st,
         static_cast<const uint8_t *>(k_new), static_cast<const uint8_t *>(v_new), keep_mask, mn, is_cond,
-        row_bytes, bk, static_cast<uint8_t *>(bank->k_store), static_cast<uint8_t *>(bank->v_store), status);
+        row_bytes, bk, static_cast<uint8_t *>(bank->k_store), static_cast<uint8_t *>(bank->v_store), status,
+        rope, bank->d, elem_bytes(bank->dtype));
     if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
     return RS3_OK;
+}
+
+}  // namespace
+
+extern "C" rs3_status rs3_bank_commit(const rs3_bank *bank, const void *k_new, const void *v_new,
+                                      const uint8_t *keep_mask, int is_cond, int32_t *status,
+                                      rs3_stream_t stream)
+{
+    return commit_launch(bank, k_new, v_new, keep_mask, is_cond, nullptr, status, stream);
+}
+
+extern "C" rs3_status rs3_bank_commit_rope(const rs3_bank *bank, const void *k_new, const void *v_new,
+                                           const uint8_t *keep_mask, int is_cond, const float *rope_cos_sin,
+                                           int32_t *status, rs3_stream_t stream)
+{
+    if (!rope_cos_sin || !rs3_aligned16(rope_cos_sin)) return RS3_EINVAL;
+    if (bank_ok(bank) && bank->d % 8 != 0) return RS3_EUNSUPPORTED;   // whole pairs in every 16-byte piece
+    return commit_launch(bank, k_new, v_new, keep_mask, is_cond, rope_cos_sin, status, stream);
 }
 
 extern "C" rs3_status rs3_bank_set_pointers(const rs3_bank *bank, const void *k_ptr,

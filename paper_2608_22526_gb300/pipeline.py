@@ -81,9 +81,14 @@ class Pipeline:
                                      stream if stream is not None else self.stream)
 
     def commit(self, k_new: torch.Tensor, v_new: torch.Tensor, mask: Optional[torch.Tensor],
-               is_cond: int):
-        rs3.rs3_bank_commit(self.bank, k_new, v_new, None if self.dense else mask, is_cond,
-                            self.status, self.stream)
+               is_cond: int, rope: Optional[torch.Tensor] = None):
+        """Eq. 8's sparse write; with a RoPE table the keys are stored rotated
+        by their own cell (Eq. 7 on the key side)."""
+        m = None if self.dense else mask
+        if rope is None:
+            rs3.rs3_bank_commit(self.bank, k_new, v_new, m, is_cond, self.status, self.stream)
+        else:
+            rs3.rs3_bank_commit_rope(self.bank, k_new, v_new, m, is_cond, rope, self.status, self.stream)
 
     def set_pointers(self, kp: torch.Tensor, vp: torch.Tensor):
         rs3.rs3_bank_set_pointers(self.bank, kp, vp, self.status, self.stream)

@@ -62,6 +62,7 @@ SIGNATURES = {
     "rs3_bank_layout": (_I, [_I, _I, _I, _I, _I, _I, _I, _I64, _I, _I, _P, _P]),
     "rs3_bank_init": (_I, [_P, _I, _I, _I, _I, _I, _I, _I, _I64, _I, _I, _P, _P, _P, _P]),
     "rs3_bank_commit": (_I, [_P, _P, _P, _P, _I, _P, _P]),
+    "rs3_bank_commit_rope": (_I, [_P, _P, _P, _P, _I, _P, _P, _P]),
     "rs3_bank_set_pointers": (_I, [_P, _P, _P, _P, _P]),
     "rs3_bank_reset": (_I, [_P, _I, _P]),
     "rs3_bank_read_meta": (_I, [_P, _P, _P, _P]),
@@ -252,6 +253,12 @@ def rs3_bank_commit(bank: Bank, k_new, v_new, keep_mask, is_cond: int, status, s
     rc = lib.rs3_bank_commit(ctypes.byref(bank.desc), _ptr(k_new), _ptr(v_new), _ptr(keep_mask),
                              int(is_cond), _ptr(status), _stream(stream))
     _check(rc, "rs3_bank_commit")
+
+
+def rs3_bank_commit_rope(bank: Bank, k_new, v_new, keep_mask, is_cond: int, rope, status, stream=None):
+    rc = lib.rs3_bank_commit_rope(ctypes.byref(bank.desc), _ptr(k_new), _ptr(v_new), _ptr(keep_mask),
+                                  int(is_cond), _ptr(rope), _ptr(status), _stream(stream))
+    _check(rc, "rs3_bank_commit_rope")
 
 
 def rs3_bank_set_pointers(bank: Bank, k_ptr, v_ptr, status, stream=None):

@@ -110,6 +110,8 @@ def test_null_arguments_are_rejected_on_host(binding):
     # an uninitialised bank descriptor is refused by every bank call
     desc = binding.BankDesc()
     assert lib.rs3_bank_commit(ctypes.byref(desc), one, one, None, 0, one, None) == binding.RS3_EINVAL
+    assert lib.rs3_bank_commit_rope(ctypes.byref(desc), one, one, None, 0, one, one, None) == binding.RS3_EINVAL
+    assert lib.rs3_bank_commit_rope(ctypes.byref(desc), one, one, None, 0, None, one, None) == binding.RS3_EINVAL
     assert lib.rs3_bank_reset(ctypes.byref(desc), -1, None) == binding.RS3_EINVAL
     assert lib.rs3_memory_readout(one, 1, 1, 4096, 1, 256, one, one, one, 1228, ctypes.byref(desc),
                                   None, None, one, 0.0, one, 1 << 30, one, None) == binding.RS3_EINVAL

@@ -59,6 +59,16 @@ def test_multistream_full_size():
                  threads=16)
 
 
+@pytest.mark.parametrize("name", ["sam2_1obj", "multistream"])
+def test_rope_on_queries_and_keys(name):
+    """Eq. 7 on both sides: queries rotated by their cell in the readout, keys
+    stored rotated by their cell at commit (pointer rows unrotated); the bank
+    holds the oracle's rotated keys to one bf16 unit and the readout matches
+    the oracle's attention over them."""
+    w = synth.scaled(W[name], frames=10)
+    run_lockstep(w, check_frames={1, 9}, rope=True, rope_keys=True, rows_per_unit=64)
+
+
 def test_multistream_rope_small():
     w = synth.scaled(W["multistream"], frames=8, G=2)
     run_lockstep(w, check_frames={1, 7}, rope=True, rows_per_unit=64)

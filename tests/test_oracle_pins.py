@@ -416,6 +416,105 @@ def test_rope_gather_equals_rotate_then_gather():
     assert np.max(np.abs(Abad - A)) > 1e-3
 
 
+def test_key_rotation_is_the_complex_product():
+    """Eq. 7 on the key side: each pair (2p, 2p+1) of every head of row i,
+    read as a complex number, times cos + i sin of the table's entry (i, p)."""
+    rng = np.random.default_rng(43)
+    mn, H, d = 12, 2, 8
+    x = rng.standard_normal((mn, H * d)).astype(np.float32)
+    tab, _ = _rope_table(mn, d, rng)
+    y = orc.rotate_rows(x, "f32", tab).astype(np.float64).reshape(mn, H, d // 2, 2)
+    f = tab[..., 0].astype(np.float64) + 1j * tab[..., 1].astype(np.float64)
+    xc = x.astype(np.float64).reshape(mn, H, d // 2, 2)
+    z = (xc[..., 0] + 1j * xc[..., 1]) * f[:, None, :]
+    assert np.max(np.abs(y[..., 0] - z.real)) < 1e-6 and np.max(np.abs(y[..., 1] - z.imag)) < 1e-6
+    # bf16 storage: the fp64 rotation rounded once to nearest-even
+    xb = orc.round_to(x.astype(np.float64), "bf16")
+    yb = orc.rotate_rows(xb, "bf16", tab)
+    xbc = orc.widen(xb, "bf16").astype(np.float64).reshape(mn, H, d // 2, 2)
+    zb = (xbc[..., 0] + 1j * xbc[..., 1]) * f[:, None, :]
+    ref = np.stack([zb.real, zb.imag], -1).reshape(mn, H * d)
+    assert np.array_equal(yb, orc.round_to(ref, "bf16"))
+
+
+def test_key_rotation_zero_angle_keeps_keys_bit_for_bit():
+    rng = np.random.default_rng(47)
+    mn, d = 9, 16
+    tab = np.zeros((mn, d // 2, 2), np.float32)
+    tab[..., 0] = 1.0
+    xb = orc.round_to(rng.standard_normal((mn, 2 * d)), "bf16")
+    assert np.array_equal(orc.rotate_rows(xb, "bf16", tab), xb)
+
+
+def test_rotated_bank_equals_rotating_keys_at_read_time():
+    """Storing keys rotated by their own cell and reading them with rotated
+    queries is the attention of Eq. 6/7 with both sides rotated at read time."""
+    rng = np.random.default_rng(53)
+    mn, H, d = 16, 2, 8
+    q = rng.standard_normal((mn, H * d)).astype(np.float32)
+    kx = rng.standard_normal((mn, H * d)).astype(np.float32)
+    V = rng.standard_normal((mn, H * d)).astype(np.float32)
+    tab, _ = _rope_table(mn, d, rng)
+    key_cells = np.array([1, 4, 5, 9, 12, 15])
+    krot = orc.rotate_rows(kx, "f32", tab)[key_cells]
+    idx = np.array([0, 3, 8, 14], np.int32)
+    A = orc.readout(q, "f32", H, d, idx, krot, V[key_cells], "f32", rope=tab)
+    f = tab[..., 0].astype(np.float64) + 1j * tab[..., 1].astype(np.float64)
+
+    def rot(x, cells):
+        xc = x.astype(np.float64).reshape(-1, H, d // 2, 2)
+        z = (xc[..., 0] + 1j * xc[..., 1]) * f[cells][:, None, :]
+        return np.stack([z.real, z.imag], -1).reshape(-1, H * d)
+    qr, kr = rot(q[idx], idx), rot(kx[key_cells], key_cells)
+    Vd = V[key_cells].astype(np.float64)
+    ref = np.zeros((idx.size, H * d))
+    for h in range(H):
+        sl = slice(h * d, (h + 1) * d)
+        s = qr[:, sl] @ kr[:, sl].T / math.sqrt(d)
+        w = np.exp(s - s.max(axis=1, keepdims=True))
+        ref[:, sl] = (w / w.sum(axis=1, keepdims=True)) @ Vd[:, sl]
+    assert np.max(np.abs(A - ref)) < 1e-5               # keys held in fp32 after their rotation
+
+
+def test_rotated_queries_and_keys_see_only_relative_positions():
+    """With a 1-D rotary table (angle = position x frequency), rotating the
+    query by its cell and the keys by theirs makes every score depend on the
+    cells' difference only: shifting all cells together leaves the attention
+    unchanged.  A sign mismatch between the two rotations would break this."""
+    rng = np.random.default_rng(59)
+    mn, d = 64, 8
+    freq = np.array([1.0, 0.31, 0.097, 0.029])
+    ang = np.arange(mn)[:, None] * freq[None, :]
+    tab = np.stack([np.cos(ang), np.sin(ang)], -1).astype(np.float64)
+    tab32 = tab.astype(np.float32)
+    qv = rng.standard_normal(d).astype(np.float32)
+    kv = rng.standard_normal((5, d)).astype(np.float32)
+    V = rng.standard_normal((5, d)).astype(np.float32)
+    outs = []
+    for shift in (0, 17, 40):
+        qcell = 3 + shift
+        kcells = np.array([0, 2, 5, 9, 20]) + shift
+        q = np.zeros((mn, d), np.float32)
+        q[qcell] = qv
+        kx = np.zeros((mn, d), np.float32)
+        kx[kcells] = kv
+        krot = orc.rotate_rows(kx, "f32", tab32)[kcells]
+        outs.append(orc.readout(q, "f32", 1, d, np.array([qcell], np.int32), krot, V, "f32", rope=tab32))
+    assert np.max(np.abs(outs[1] - outs[0])) < 1e-5 and np.max(np.abs(outs[2] - outs[0])) < 1e-5
+    # keys rotated the opposite way do not have the property
+    bad = np.stack([tab32[..., 0], -tab32[..., 1]], -1)
+    outs_bad = []
+    for shift in (0, 17):
+        qcell, kcells = 3 + shift, np.array([0, 2, 5, 9, 20]) + shift
+        q = np.zeros((mn, d), np.float32)
+        q[qcell] = qv
+        kx = np.zeros((mn, d), np.float32)
+        kx[kcells] = kv
+        outs_bad.append(orc.readout(q, "f32", 1, d, np.array([qcell], np.int32),
+                                    orc.rotate_rows(kx, "f32", bad)[kcells], V, "f32", rope=tab32))
+    assert np.max(np.abs(outs_bad[1] - outs_bad[0])) > 1e-3
+
+
 def test_rope_zero_angle_is_identity():
     rng = np.random.default_rng(41)
     mn, d = 10, 8
