@@ -366,6 +366,33 @@ rs3_status rs3_memory_readout_merge(const void *q, rs3_dtype dtype, int G, int m
                                     void *workspace, size_t workspace_bytes, int32_t *status,
                                     rs3_stream_t stream);
 
+/*
+ * rs3_memory_readout_attend split in its two launches, with the same
+ * arguments (Sec. 3.1, Eq. 6):
+ *   rs3_memory_readout_plan  the pass-through of unselected cells (out of
+ *                            place only) and the work list in `workspace`:
+ *                            the bank's row ranges from its counters and the
+ *                            split of the work over the SMs;
+ *   rs3_memory_readout_run   the attention kernel over that work list.
+ * plan then run on one stream is exactly rs3_memory_readout_attend.  run
+ * reads the bank's rows but not its counters, so the work list describes the
+ * bank as it was when plan ran; ordering is the caller's (run after plan, and
+ * no commit to the bank between them).  Separate calls let a caller time or
+ * schedule the attention kernel on its own.
+ */
+rs3_status rs3_memory_readout_plan(const void *q, rs3_dtype dtype, int G, int mn, int H, int d,
+                                   const int32_t *unit_group, const int32_t *idx,
+                                   const int32_t *count, int k_max, const rs3_bank *bank,
+                                   const float *rope, const void *residual, void *out, float scale,
+                                   void *workspace, size_t workspace_bytes, int32_t *status,
+                                   rs3_stream_t stream);
+rs3_status rs3_memory_readout_run(const void *q, rs3_dtype dtype, int G, int mn, int H, int d,
+                                  const int32_t *unit_group, const int32_t *idx,
+                                  const int32_t *count, int k_max, const rs3_bank *bank,
+                                  const float *rope, const void *residual, void *out, float scale,
+                                  void *workspace, size_t workspace_bytes, int32_t *status,
+                                  rs3_stream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* Write side: keep-set (Sec. 3.2; Eq. 8)                                    */
 /* ------------------------------------------------------------------------ */

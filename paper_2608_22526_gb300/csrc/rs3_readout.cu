@@ -781,8 +781,8 @@ rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, in
 
 namespace {
 
-// pass-through of the unselected cells (out of place only), plan, attention
-rs3_status launch_attend(const ReadoutArgs &a, const ReadoutPath &p, rs3_dtype dtype, cudaStream_t st)
+// pass-through of the unselected cells (out of place only) and the plan
+rs3_status launch_plan(const ReadoutArgs &a, cudaStream_t st, rs3_dtype dtype)
 {
     if (a.residual != a.out) {
         const int64_t nvec = (int64_t)a.U * a.mn * a.D * (dtype == RS3_BF16 ? 2 : 4) / 16;
@@ -797,7 +797,12 @@ rs3_status launch_attend(const ReadoutArgs &a, const ReadoutPath &p, rs3_dtype d
     const size_t plan_smem = (size_t)(2 * a.U + 1) * 8 + (size_t)(3 * a.U + 1) * 4;
     if (rs3_kernel_smem((const void *)k_plan, plan_smem) != RS3_OK) return RS3_EUNSUPPORTED;
     launch_pdl(k_plan, dim3(1), dim3(PLAN_THREADS), plan_smem, st, a);
-    if (cudaGetLastError() != cudaSuccess) return RS3_ECUDA;
+    return cudaGetLastError() != cudaSuccess ? RS3_ECUDA : RS3_OK;
+}
+
+// the attention kernel over the plan in the workspace
+rs3_status launch_run(const ReadoutArgs &a, const ReadoutPath &p, rs3_dtype dtype, cudaStream_t st)
+{
     if (p.kind == 1) return rs3_launch_tc_readout(a, st);
     const size_t smem = (size_t)2 * SIMT_BN * a.d * sizeof(float);
     const int threads = 2 * a.d;
@@ -838,8 +843,12 @@ rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_
                               int64_t max_combine, rs3_dtype dtype, cudaStream_t st, int phases)
 {
     (void)max_items;
-    if (phases & RS3_PHASE_ATTEND) {
-        const rs3_status s = launch_attend(a, p, dtype, st);
+    if (phases & RS3_PHASE_PLAN) {
+        const rs3_status s = launch_plan(a, st, dtype);
+        if (s != RS3_OK) return s;
+    }
+    if (phases & RS3_PHASE_RUN) {
+        const rs3_status s = launch_run(a, p, dtype, st);
         if (s != RS3_OK) return s;
     }
     if (phases & RS3_PHASE_MERGE) return launch_merge(a, max_combine, dtype, st);
@@ -885,6 +894,28 @@ extern "C" rs3_status rs3_memory_readout_attend(const void *q, rs3_dtype dtype, 
 {
     return readout_call(q, dtype, G, mn, H, d, unit_group, idx, count, k_max, bank, rope, residual, out, scale,
                         workspace, workspace_bytes, status, stream, RS3_PHASE_ATTEND);
+}
+
+extern "C" rs3_status rs3_memory_readout_plan(const void *q, rs3_dtype dtype, int G, int mn, int H,
+                                              int d, const int32_t *unit_group, const int32_t *idx,
+                                              const int32_t *count, int k_max, const rs3_bank *bank,
+                                              const float *rope, const void *residual, void *out,
+                                              float scale, void *workspace, size_t workspace_bytes,
+                                              int32_t *status, rs3_stream_t stream)
+{
+    return readout_call(q, dtype, G, mn, H, d, unit_group, idx, count, k_max, bank, rope, residual, out, scale,
+                        workspace, workspace_bytes, status, stream, RS3_PHASE_PLAN);
+}
+
+extern "C" rs3_status rs3_memory_readout_run(const void *q, rs3_dtype dtype, int G, int mn, int H,
+                                             int d, const int32_t *unit_group, const int32_t *idx,
+                                             const int32_t *count, int k_max, const rs3_bank *bank,
+                                             const float *rope, const void *residual, void *out,
+                                             float scale, void *workspace, size_t workspace_bytes,
+                                             int32_t *status, rs3_stream_t stream)
+{
+    return readout_call(q, dtype, G, mn, H, d, unit_group, idx, count, k_max, bank, rope, residual, out, scale,
+                        workspace, workspace_bytes, status, stream, RS3_PHASE_RUN);
 }
 
 extern "C" rs3_status rs3_memory_readout_merge(const void *q, rs3_dtype dtype, int G, int mn, int H,

@@ -56,7 +56,7 @@ rs3_status rs3_readout_prepare(const void *q, rs3_dtype dtype, int G, int mn, in
                                ReadoutPath *path, int64_t *grid_items, int64_t *grid_combine);
 // phases of a readout: the attention over the bank (pass-through, plan,
 // readout kernel) and the merge of split-KV partials
-enum { RS3_PHASE_ATTEND = 1, RS3_PHASE_MERGE = 2 };
+enum { RS3_PHASE_PLAN = 1, RS3_PHASE_RUN = 4, RS3_PHASE_ATTEND = 1 | 4, RS3_PHASE_MERGE = 2 };
 rs3_status rs3_readout_launch(const ReadoutArgs &a, const ReadoutPath &p, int64_t max_items,
                               int64_t max_combine, rs3_dtype dtype, cudaStream_t st, int phases);
 

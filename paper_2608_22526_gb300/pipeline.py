@@ -71,6 +71,24 @@ class Pipeline:
                                       self.ws_readout, self.status,
                                       stream if stream is not None else self.stream)
 
+    def readout_plan(self, q: torch.Tensor, residual: Optional[torch.Tensor], out: torch.Tensor,
+                     rope: Optional[torch.Tensor] = None, scale: float = 0.0, stream=None):
+        """First launch of readout_attend(): the pass-through and the work list."""
+        w = self.w
+        rs3.rs3_memory_readout_plan(q, w.dtype, w.G, w.mn, w.H, w.d, self.unit_group, self.idx,
+                                    self.count, self.k_max, self.bank, rope, residual, out, scale,
+                                    self.ws_readout, self.status,
+                                    stream if stream is not None else self.stream)
+
+    def readout_run(self, q: torch.Tensor, residual: Optional[torch.Tensor], out: torch.Tensor,
+                    rope: Optional[torch.Tensor] = None, scale: float = 0.0, stream=None):
+        """Second launch of readout_attend(): the attention kernel alone."""
+        w = self.w
+        rs3.rs3_memory_readout_run(q, w.dtype, w.G, w.mn, w.H, w.d, self.unit_group, self.idx,
+                                   self.count, self.k_max, self.bank, rope, residual, out, scale,
+                                   self.ws_readout, self.status,
+                                   stream if stream is not None else self.stream)
+
     def readout_merge(self, q: torch.Tensor, residual: Optional[torch.Tensor], out: torch.Tensor,
                       rope: Optional[torch.Tensor] = None, scale: float = 0.0, stream=None):
         """Second phase of readout(): the split-KV merge; reads no bank."""

@@ -73,6 +73,10 @@ SIGNATURES = {
                                 ctypes.c_float, _P, _SZ, _P, _P]),
     "rs3_memory_readout_merge": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P, _P, _P, _P,
                                 ctypes.c_float, _P, _SZ, _P, _P]),
+    "rs3_memory_readout_plan": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P, _P, _P, _P,
+                                ctypes.c_float, _P, _SZ, _P, _P]),
+    "rs3_memory_readout_run": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P, _P, _P, _P,
+                                ctypes.c_float, _P, _SZ, _P, _P]),
     "rs3_set_wait_limit_ns": (None, [ctypes.c_uint64]),
     "rs3_get_wait_limit_ns": (ctypes.c_uint64, []),
     "rs3_write_keepset": (_I, [_P, _P, _I, _I, _I, _P, _P, _P, _P]),
@@ -188,6 +192,20 @@ def rs3_memory_readout_attend(q, dtype: str, G: int, mn: int, H: int, d: int, un
                               k_max: int, bank: "Bank", rope, residual, out, scale: float, workspace,
                               status, stream=None):
     _readout_phase(lib.rs3_memory_readout_attend, "rs3_memory_readout_attend", q, dtype, G, mn, H, d,
+                   unit_group, idx, count, k_max, bank, rope, residual, out, scale, workspace, status, stream)
+
+
+def rs3_memory_readout_plan(q, dtype: str, G: int, mn: int, H: int, d: int, unit_group, idx, count,
+                            k_max: int, bank: "Bank", rope, residual, out, scale: float, workspace,
+                            status, stream=None):
+    _readout_phase(lib.rs3_memory_readout_plan, "rs3_memory_readout_plan", q, dtype, G, mn, H, d,
+                   unit_group, idx, count, k_max, bank, rope, residual, out, scale, workspace, status, stream)
+
+
+def rs3_memory_readout_run(q, dtype: str, G: int, mn: int, H: int, d: int, unit_group, idx, count,
+                           k_max: int, bank: "Bank", rope, residual, out, scale: float, workspace,
+                           status, stream=None):
+    _readout_phase(lib.rs3_memory_readout_run, "rs3_memory_readout_run", q, dtype, G, mn, H, d,
                    unit_group, idx, count, k_max, bank, rope, residual, out, scale, workspace, status, stream)
 
 
