@@ -244,8 +244,10 @@ def run_step(pipe, data, timers=None, side=None, merge=None, att_ev=None):
     every SM), with "readout" beside the readout and commit, with "none" in
     line on the main stream.  With SPLIT_MERGE the readout runs as its two
     phases: the attention on the main stream, the split-KV merge on `merge`
-    beside the frame's commit (the merge reads no bank); the next attention
-    waits for the merge, which shares its workspace.  With `att_ev` (a list)
+    beside the frame's commit and the next frames' work (the merge reads no
+    bank).  Frame t uses keep-set buffer and readout workspace t % 2, so the
+    attention of frame t waits only for the merge of frame t - 2, the last
+    reader of its workspace.  With `att_ev` (a list)
     every frame's attention phase is bracketed by a pair of timing events
     that become event nodes when the step is captured in a graph."""
     import torch
@@ -298,8 +300,8 @@ def run_step(pipe, data, timers=None, side=None, merge=None, att_ev=None):
         if t + 1 < data.T and OVERLAP == "readout":
             issue_select(t + 1)          # beside this frame's readout and commit
         main.wait_event(sel_ev[t])
-        if t - 1 in rd_ev and mrg is not main:
-            main.wait_event(rd_ev[t - 1])   # the previous merge still reads the workspace
+        if t - 2 in rd_ev and mrg is not main:
+            main.wait_event(rd_ev[t - 2])   # the merge of t - 2 read this workspace
         pipe.use_buffer(t % 2)
         if timers is not None:
             e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]

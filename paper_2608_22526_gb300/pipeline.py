@@ -36,8 +36,11 @@ class Pipeline:
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
         self.ws_select = torch.empty(rs3.rs3_select_workspace_bytes(w.G, w.U, w.m, w.n),
                                      dtype=torch.uint8, device=dev)
-        self.ws_readout = torch.empty(rs3.rs3_readout_workspace_bytes(w.U, w.H, w.d, self.k_max, w.dtype),
-                                      dtype=torch.uint8, device=dev)
+        # two readout workspaces, paired with the keep-set buffers: the merge of
+        # frame t reads its workspace while frame t+1 plans and attends in the other
+        nws = rs3.rs3_readout_workspace_bytes(w.U, w.H, w.d, self.k_max, w.dtype)
+        self.ws_buf = [torch.empty(nws, dtype=torch.uint8, device=dev) for _ in range(2)]
+        self.ws_readout = self.ws_buf[0]
         if ring_cap is None:
             ring_cap = w.ring_cap_rows() if (dense or w.window > 0) else w.ring_cap_rows_tight()
         self.bank = rs3.Bank(w.U, w.H, w.d, w.dtype, w.mn, w.n_cond, w.window, ring_cap,
@@ -46,8 +49,10 @@ class Pipeline:
 
     # -- library calls -------------------------------------------------------
     def use_buffer(self, i: int):
-        """Selects which keep-set buffer the next select / readout use."""
+        """Selects which keep-set buffer (and readout workspace) the next
+        select / readout use."""
         self.idx, self.count = self.idx_buf[i], self.count_buf[i]
+        self.ws_readout = self.ws_buf[i]
 
     def select(self, z: torch.Tensor, prev_masks: torch.Tensor, stream=None):
         w = self.w
