@@ -235,7 +235,7 @@ OVERLAP = "readout"
 SPLIT_MERGE = True
 
 
-def run_step(pipe, data, timers=None, side=None, merge=None, att_ev=None):
+def run_step(pipe, data, side=None, merge=None, att_ev=None):
     """One step: the whole sequence through the library (Algorithm 1's loop).
 
     The selection of frame t+1 needs only frame t+1's grid and frame t's mask,
@@ -247,25 +247,23 @@ def run_step(pipe, data, timers=None, side=None, merge=None, att_ev=None):
     beside the frame's commit and the next frames' work (the merge reads no
     bank).  Frame t uses keep-set buffer and readout workspace t % 2, so the
     attention of frame t waits only for the merge of frame t - 2, the last
-    reader of its workspace.  With `att_ev` (a list)
-    every frame's attention phase is bracketed by a pair of timing events
-    that become event nodes when the step is captured in a graph."""
+    reader of its workspace.  Without `side` and `merge` every call runs in
+    line on the main stream, the readout as one call.  With `att_ev` (a list)
+    every frame's attention phase is bracketed by timing events that become
+    event nodes when the step is captured in a graph."""
     import torch
     w = pipe.w
     from paper_2608_22526_gb300 import rs3
     main = torch.cuda.current_stream()
     side = side if (side is not None and OVERLAP != "none") else main
-    # the per-call timing pass (timers) issues each frame's calls back to back
-    # on one stream, the readout as one call, so that their event times are
-    # the calls' own durations
-    mrg = merge if (merge is not None and SPLIT_MERGE and timers is None) else main
+    mrg = merge if (merge is not None and SPLIT_MERGE) else main
     rs3.rs3_bank_reset(pipe.bank, -1)
     pipe.track.zero_()
     F = data.frame
     fork = torch.cuda.Event()
     fork.record(main)
     side.wait_event(fork)
-    sel_ev, rd_ev, sel_t = {}, {}, {}
+    sel_ev, rd_ev = {}, {}
 
     def issue_select(t, after=None):
         # frame t's keep-set goes to buffer t % 2, last read by the readout of t - 2
@@ -274,15 +272,10 @@ def run_step(pipe, data, timers=None, side=None, merge=None, att_ev=None):
         if after is not None:
             side.wait_event(after)
         pipe.use_buffer(t % 2)
-        if timers is not None:
-            sel_t[t] = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
-            sel_t[t][0].record(side)
         pipe.select(F("z", t), F("prev", t), stream=side)
-        ev = torch.cuda.Event(enable_timing=timers is not None)
+        ev = torch.cuda.Event()
         ev.record(side)
         sel_ev[t] = ev
-        if timers is not None:
-            sel_t[t][1] = ev
 
     rope = getattr(data, "rope", None)
     first = data.P + (1 if w.n_cond > 0 else 0)
@@ -299,25 +292,25 @@ def run_step(pipe, data, timers=None, side=None, merge=None, att_ev=None):
             issue_select(t)
         if t + 1 < data.T and OVERLAP == "readout":
             issue_select(t + 1)          # beside this frame's readout and commit
+        # the selection of frame t waited for the merge of frame t - 2, the last
+        # reader of this frame's keep-set buffer and workspace, so this one wait
+        # orders the readout after both (a second edge, straight from the merge
+        # branch, let the graph queue the plan behind the merge of frame t - 1)
         main.wait_event(sel_ev[t])
-        if t - 2 in rd_ev and mrg is not main:
-            main.wait_event(rd_ev[t - 2])   # the merge of t - 2 read this workspace
         pipe.use_buffer(t % 2)
-        if timers is not None:
-            e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
-            e[0].record(main)
         if mrg is main:
             pipe.readout(F("z", t), F("x", t), F("x", t), rope=rope)   # both phases, one call
         else:
             if att_ev is not None:
                 # the attend phase as its two launches, with an event between
                 # them: the plan, then the attention kernel on its own
-                ea = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(3)]
+                ea = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)]
                 ea[0].record(main)
                 pipe.readout_plan(F("z", t), F("x", t), F("x", t), rope=rope)
                 ea[1].record(main)
                 pipe.readout_run(F("z", t), F("x", t), F("x", t), rope=rope)
                 ea[2].record(main)
+                ea[3].record(main)       # an empty interval: the event nodes' own cost
                 att_ev.append(ea)
             else:
                 pipe.readout_attend(F("z", t), F("x", t), F("x", t), rope=rope)
@@ -325,18 +318,12 @@ def run_step(pipe, data, timers=None, side=None, merge=None, att_ev=None):
             att.record(main)
             mrg.wait_event(att)
             pipe.readout_merge(F("z", t), F("x", t), F("x", t), rope=rope, stream=mrg)
-        ev = torch.cuda.Event(enable_timing=timers is not None)
+        ev = torch.cuda.Event()
         ev.record(mrg)
         rd_ev[t] = ev                        # frame t's keep-set and workspace are free
         if t + 1 < data.T and OVERLAP != "readout":
             issue_select(t + 1, after=ev)    # beside this frame's commit
-        if timers is not None:
-            e[1] = ev
-            e[2].record(main)
         pipe.commit(F("k", t), F("v", t), F("mask", t), 0, rope=rope)
-        if timers is not None:
-            e[3].record(main)
-            timers.append((t, [sel_t[t][0], sel_t[t][1], e[0], e[1], e[2], e[3]]))
     for st in (side, mrg):
         if st is not main:
             join = torch.cuda.Event()
@@ -344,12 +331,37 @@ def run_step(pipe, data, timers=None, side=None, merge=None, att_ev=None):
             main.wait_event(join)
 
 
+def calls_only(pipe, data, what):
+    """One kind of call of the pass alone, back to back on the current stream:
+    "select" -- every readout frame's selection; "commit" -- every commit of
+    the pass (prefill, conditioning frame, readout frames) from an empty bank;
+    "setup" -- only the commits before the first readout frame."""
+    from paper_2608_22526_gb300 import rs3
+    w = pipe.w
+    F = data.frame
+    rope = getattr(data, "rope", None)
+    rs3.rs3_bank_reset(pipe.bank, -1)
+    pipe.track.zero_()
+    for t in range(data.T):
+        setup = t < data.P or (t == data.P and w.n_cond > 0)
+        if what == "select":
+            if not setup:
+                pipe.use_buffer(t % 2)
+                pipe.select(F("z", t), F("prev", t))
+        elif setup or what == "commit":
+            mask = None if t < data.P else F("mask", t)
+            pipe.commit(F("k", t), F("v", t), mask, int(t == data.P and w.n_cond > 0), rope=rope)
+
+
 def frame_work(w, counts, bank_lens, kw_lens):
     """Algorithmic flops and bytes of one frame from the selected sizes."""
     b = 2 if w.dtype == "bf16" else 4
     flops = sum(4.0 * c * n * w.H * w.d for c, n in zip(counts, bank_lens))
     commit_bytes = w.U * w.mn + sum(4.0 * L * w.D * b for L in kw_lens)
-    return flops, commit_bytes
+    # selection: the grids z (one per group), the previous masks, the keep-set
+    # written, the counts and the tracker state read and written
+    select_bytes = w.G * w.mn * w.D * b + w.U * w.mn + 4.0 * sum(counts) + 4 * w.U + 2 * 24 * w.U
+    return flops, commit_bytes, select_bytes
 
 
 def work_model(pipe, data):
@@ -437,32 +449,56 @@ def gpu_arm(args):
             torch.cuda.synchronize()
             work = work_model(pipe, data)
             torch.cuda.synchronize()
-            # per-call timing pass (events on each call's launching stream)
-            timers = []
-            run_step(pipe, data, timers, side=side, merge=merge)
-            torch.cuda.synchronize()
-            sel_ms = [t[1][0].elapsed_time(t[1][1]) for t in timers]
-            call_ms = [t[1][2].elapsed_time(t[1][3]) for t in timers]
-            cm_ms = [t[1][4].elapsed_time(t[1][5]) for t in timers]
+            # per-call times: graphs of one kind of call alone (the pass's
+            # selections; its commits; the commits before the first readout
+            # frame) and of the whole pass with every call in line on one
+            # stream, each timed over whole replays with no event node inside
+            # (an event node adds about 5 us to the interval it brackets)
+            def graph_us(fn, n=5):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=stream):
+                    fn()
+                for _ in range(3):
+                    g.replay()
+                torch.cuda.synchronize()
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record()
+                for _ in range(n):
+                    g.replay()
+                b.record()
+                torch.cuda.synchronize()
+                del g
+                return a.elapsed_time(b) * 1e3 / n
+            n_fr = len(work)
+            t_serial = graph_us(lambda: run_step(pipe, data))
+            t_sel = graph_us(lambda: calls_only(pipe, data, "select"))
+            t_cm = graph_us(lambda: calls_only(pipe, data, "commit"))
+            t_setup = graph_us(lambda: calls_only(pipe, data, "setup"))
+            sel_us = t_sel / n_fr
+            cm_us = max(t_cm - t_setup, 0.0) / n_fr
+            call_us = max(t_serial - t_sel - t_cm, 0.0) / n_fr
             graph = torch.cuda.CUDAGraph()
             with torch.cuda.graph(graph, stream=stream):
                 run_step(pipe, data, side=side, merge=merge)
             # the attention phase of every frame timed inside a graph of the
             # same sequence (event nodes around each attend call)
-            att_ms = run_ms = None
+            att_ms = run_ms = empty_ms = None
             if SPLIT_MERGE and _events_supported():
                 att_ev = []
                 g_att = torch.cuda.CUDAGraph()
                 with torch.cuda.graph(g_att, stream=stream):
                     run_step(pipe, data, side=side, merge=merge, att_ev=att_ev)
-                per, per_run = [], []
+                per, per_run, per_empty = [], [], []
                 for _ in range(3):
                     g_att.replay()
                     torch.cuda.synchronize()
-                    per.append([a.elapsed_time(c) for a, b, c in att_ev])
-                    per_run.append([b.elapsed_time(c) for a, b, c in att_ev])
+                    per.append([a.elapsed_time(c) for a, b, c, _ in att_ev])
+                    per_run.append([b.elapsed_time(c) for a, b, c, _ in att_ev])
+                    per_empty.append([c.elapsed_time(d) for a, b, c, d in att_ev])
                 att_ms = list(np.mean(np.array(per[1:]), axis=0))
                 run_ms = list(np.mean(np.array(per_run[1:]), axis=0))
+                empty_ms = float(np.median(np.array(per_empty[1:])))
                 del g_att
             # passes per step
             for _ in range(args.warmup):
@@ -552,8 +588,10 @@ def gpu_arm(args):
                 del graph2, twin
         flops = [frame_work(w, c, n, k)[0] for (_, c, n, k) in work]
         cbytes = [frame_work(w, c, n, k)[1] for (_, c, n, k) in work]
-        results[mode] = dict(dev_s=dev_s, e2e_s=e2e_s, clocks=clk, sel_ms=sel_ms, call_ms=call_ms,
-                             att_ms=att_ms, run_ms=run_ms, cm_ms=cm_ms, flops=flops, cbytes=cbytes,
+        sbytes = [frame_work(w, c, n, k)[2] for (_, c, n, k) in work]
+        results[mode] = dict(dev_s=dev_s, e2e_s=e2e_s, clocks=clk, sel_us=sel_us, call_us=call_us,
+                             att_ms=att_ms, run_ms=run_ms, empty_ms=empty_ms, cm_us=cm_us, flops=flops, cbytes=cbytes,
+                             sbytes=sbytes,
                              e2e_passes=e2e_passes if mode == "pruned" and e2e_s else None,
                              e2e_bytes=e2e_bytes if mode == "pruned" and e2e_s else None,
                              counts=[c for (_, c, _, _) in work], lens=[n for (_, _, n, _) in work])
@@ -605,13 +643,18 @@ def gpu_arm(args):
             "us_per_launch": round(run_s / len(P["run_ms"]) * 1e6, 3),
             "peak_source": f"bf16_tflops burst, {peak_src}",
             "attend_us_per_frame": round(att_s / len(P["att_ms"]) * 1e6, 3),
-            "attend": "rs3_memory_readout_attend = " + ATTEND_KERNELS + ", events around plan and run"}
+            "attend": "rs3_memory_readout_attend = " + ATTEND_KERNELS + ", events around plan and run",
+            "empty_event_interval_us": round(P["empty_ms"] * 1e3, 3),
+            "event_note": "us_per_launch is the interval between event nodes around the launch, so it "
+                          "includes the event nodes' own cost (a graph node pair around a tiny kernel "
+                          "reads about 5 us); frac is not corrected for it"}
         line["readout_tflops"] = round(achieved, 3)
     line.update({
-        "commit_gbs": round(float(np.sum(P["cbytes"])) / (float(np.sum(P["cm_ms"])) / 1e3) / 1e9, 2),
-        "select_ms": round(float(np.mean(P["sel_ms"])), 4),
-        "readout_call_ms": round(float(np.mean(P["call_ms"])), 4),
-        "commit_ms": round(float(np.mean(P["cm_ms"])), 4),
+        "commit_gbs": round(float(np.mean(P["cbytes"])) / (P["cm_us"] / 1e6) / 1e9, 2),
+        "select_ms": round(P["sel_us"] / 1e3, 4),
+        "select_gbs": round(float(np.mean(P["sbytes"])) / (P["sel_us"] / 1e6) / 1e9, 2),
+        "readout_call_ms": round(P["call_us"] / 1e3, 4),
+        "commit_ms": round(P["cm_us"] / 1e3, 4),
         "mean_queries": round(float(np.mean([sum(c) for c in P["counts"]])), 1),
         "mean_bank_rows": round(float(np.mean([sum(n) for n in P["lens"]])), 1),
         "bank": bank_summary(w, P["lens"], results.get("dense", {}).get("lens")),
@@ -619,8 +662,12 @@ def gpu_arm(args):
         "gpu_launches": launches_per_pass(w) * reps * args.steps,
     })
     line["commit_frac_hbm"] = round(line["commit_gbs"] / hbm, 4)
-    line["per_call_note"] = ("select_ms, readout_call_ms and commit_ms are CUDA-event times of each "
-                             "call issued on its own outside the graph (host launch included)")
+    line["select_frac_hbm"] = round(line["select_gbs"] / hbm, 4)
+    line["per_call_note"] = ("select_ms and commit_ms: a CUDA graph of the pass's selections alone (its "
+                             "commits alone, less the commits before the first readout frame) over the "
+                             "readout frames; readout_call_ms: the pass with every call in line on one "
+                             "stream less those two; whole replays timed, no event node inside; GB/s = "
+                             "algorithmic bytes over those times")
     if "rope" in results:
         Rn = results["rope"]
         rope_fps = frames_per_pass * reps * args.steps / Rn["dev_s"]

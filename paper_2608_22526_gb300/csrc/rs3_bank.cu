@@ -3,7 +3,9 @@
 //
 // A commit is one launch (k_commit): a CTA per (128-cell chunk, unit) ranks
 // its kept cells with ballot/popc and copies their K and V rows with 128-bit
-// accesses; the last CTA of each unit publishes the new counters.
+// accesses, the first rows' loads in flight while the unit's counts and the
+// capacity decision are made; the last CTA of each unit publishes the new
+// counters.
 #include "rs3_internal.cuh"
 
 #include <cstdlib>
@@ -82,154 +84,204 @@ __device__ __forceinline__ int nonzero_bytes(uint4 w)
 }
 
 // The commit of one frame, in one launch: CTA (c, u) owns cells
-// [c * COMMIT_CHUNK, (c+1) * COMMIT_CHUNK) of unit u.  Every CTA reads the
-// unit's old counters, counts the unit's kept rows (and those before its
-// chunk), takes the same eviction / capacity decision, ranks its kept cells
-// with ballot/popc and copies their K and V rows as 16-byte pieces spread
-// over all its threads.  The last CTA of the unit to finish (an arrival
-// count in the unit's metadata, after a fence) publishes the new counters and
-// the frame-table entry, so no CTA can see counters of the frame it copies.
-__global__ void __launch_bounds__(256)
+// [c * CHUNK, (c+1) * CHUNK) of unit u, one cell per thread (CHUNK = 128, or
+// 64 where 128-cell chunks would give fewer than two CTAs per SM).
+// Its latency chain is two memory round trips: (1) the chunk's own mask bytes
+// and the unit's whole mask row (the kept rows before the chunk and in the
+// unit) are loaded together; (2) as soon as the chunk's kept cells are ranked
+// (ballot / popc) their first K and V pieces are loaded into registers, and
+// the unit's counts and the eviction / capacity decision (thread 0, from the
+// old counters) are made while those loads are in flight; then the pieces
+// are stored at their ring rows.  Every CTA arrives on the unit's counter
+// once thread 0 has read the old counters, and the last to arrive publishes
+// the new ones after its own stores, so no CTA can read counters of the frame
+// it copies (the readers of the bank are later launches).
+constexpr int COMMIT_PF = 8;        // kept rows per warp and batch (one piece per lane and row)
+
+// Loads piece v of rows j0, j0 + NW, ... of the chunk's kept list (NW warps).
+template <int NW>
+__device__ __forceinline__ void commit_load(uint4 (&kk)[COMMIT_PF], uint4 (&vv)[COMMIT_PF],
+                                            const int32_t *s_list, int nk, int j0, int v, int nvec,
+                                            const uint8_t *ksrc, const uint8_t *vsrc, int64_t row_bytes)
+{
+#pragma unroll
+    for (int r = 0; r < COMMIT_PF; ++r) {
+        const int j = j0 + NW * r;
+        if (j < nk && v < nvec) {
+            const int64_t so = (int64_t)s_list[j] * row_bytes + 16 * v;
+            kk[r] = __ldcs(reinterpret_cast<const uint4 *>(ksrc + so));
+            vv[r] = __ldcs(reinterpret_cast<const uint4 *>(vsrc + so));
+        }
+    }
+}
+
+// Stores those pieces at bank row row0 + j (a ring position, wrapped once,
+// past the pinned region; or a pinned row for a conditioning frame).
+template <int NW, bool ROPE>
+__device__ __forceinline__ void commit_store(const uint4 (&kk)[COMMIT_PF], const uint4 (&vv)[COMMIT_PF],
+                                             const int32_t *s_list, int nk, int j0, int v, int nvec,
+                                             int64_t row0, int is_cond, const BankDev &bk,
+                                             uint8_t *kdst, uint8_t *vdst, int64_t row_bytes,
+                                             const float *rope, int d, int esz)
+{
+#pragma unroll
+    for (int r = 0; r < COMMIT_PF; ++r) {
+        const int j = j0 + NW * r;
+        if (j < nk && v < nvec) {
+            int64_t row = row0 + j;
+            if (!is_cond) row = bk.pinned_cap + (row >= bk.ring_cap ? row - bk.ring_cap : row);
+            const int64_t dst = row * row_bytes + 16 * v;
+            uint4 k = kk[r];
+            if (ROPE) {                                    // keys stored rotated by their own cell
+                const int e = (16 * v) / esz;              // first element of the piece
+                k = rotate_piece(k, rope + ((int64_t)s_list[j] * (d / 2) + (e % d) / 2) * 2, esz);
+            }
+            *reinterpret_cast<uint4 *>(kdst + dst) = k;
+            *reinterpret_cast<uint4 *>(vdst + dst) = vv[r];
+        }
+    }
+}
+
+template <int CHUNK, bool ROPE>
+__global__ void __launch_bounds__(CHUNK)
 k_commit(const uint8_t *__restrict__ k_new, const uint8_t *__restrict__ v_new,
          const uint8_t *__restrict__ mask, int mn, int is_cond, int64_t row_bytes, BankDev bk,
          uint8_t *__restrict__ k_store, uint8_t *__restrict__ v_store, int32_t *status,
          const float *__restrict__ rope, int d, int esz)
 {
+    constexpr int NW = CHUNK / 32;
     pdl_wait();
-    __shared__ int32_t s_list[COMMIT_CHUNK];
-    __shared__ int64_t s_row[COMMIT_CHUNK];
-    __shared__ int32_t s_red[2][8];
-    __shared__ int s_last;
+    __shared__ int32_t s_list[CHUNK];
+    __shared__ int32_t s_wc[NW];
+    __shared__ int32_t s_red[2][NW];
+    __shared__ int64_t s_row0;
+    __shared__ int s_ok;
     const int u = blockIdx.y, ch = blockIdx.x;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int c0 = ch * CHUNK;
     int64_t *mu = bk.meta + (int64_t)u * bk.stride_words;
     const uint8_t *Mu = mask ? mask + (size_t)u * mn : nullptr;
-    const int64_t head0 = mu[BM_HEAD], tail0 = mu[BM_TAIL];
-    const int64_t nf0 = mu[BM_NFRAMES], oldest0 = mu[BM_OLDEST];
-    const int64_t cond_len0 = mu[BM_COND_LEN], ncond0 = mu[BM_NCOND];
-    const int64_t *foff = mu + BM_HEADER_WORDS;
-    const int64_t *flen = foff + bk.max_frames;
 
-    // kept rows of the whole unit, and of the chunks before this one
+    // the unit's old counters (thread 0 decides for the CTA)
+    int64_t head0 = 0, tail0 = 0, nf0 = 0, oldest0 = 0, cond_len0 = 0, ncond0 = 0;
+    if (threadIdx.x == 0) {
+        head0 = mu[BM_HEAD]; tail0 = mu[BM_TAIL];
+        nf0 = mu[BM_NFRAMES]; oldest0 = mu[BM_OLDEST];
+        cond_len0 = mu[BM_COND_LEN]; ncond0 = mu[BM_NCOND];
+    }
+
+    // round trip 1: this thread's cell, and the kept rows of the unit and of
+    // the chunks before this one (16-byte loads when the unit's mask row is
+    // aligned, bytes for the rest)
+    const int cell = c0 + threadIdx.x;
+    const bool keep = cell < mn && (Mu ? Mu[cell] != 0 : true);
     int total = 0, before = 0;
     if (Mu) {
-        // 16-byte loads when the unit's mask row is aligned, bytes for the rest
         const int nvec16 = (reinterpret_cast<uintptr_t>(Mu) & 15u) == 0 ? (mn >> 4) : 0;
-        for (int i = threadIdx.x; i < nvec16; i += blockDim.x) {
+#pragma unroll 4
+        for (int i = threadIdx.x; i < nvec16; i += CHUNK) {
             const int c = nonzero_bytes(__ldg(reinterpret_cast<const uint4 *>(Mu) + i));
             total += c;
-            if (i * 16 < ch * COMMIT_CHUNK) before += c;
+            before += i * 16 < c0 ? c : 0;
         }
-        for (int i = nvec16 * 16 + threadIdx.x; i < mn; i += blockDim.x) {
+        for (int i = nvec16 * 16 + threadIdx.x; i < mn; i += CHUNK) {
             const int c = Mu[i] != 0;
             total += c;
-            if (i < ch * COMMIT_CHUNK) before += c;
+            before += i < c0 ? c : 0;
         }
-    } else if (threadIdx.x == 0) {
-        total = mn;
-        before = ch * COMMIT_CHUNK;
     }
-    total = warp_sum(total);
-    before = warp_sum(before);
-    if (lane == 0) { s_red[0][warp] = total; s_red[1][warp] = before; }
-    __syncthreads();
-    int64_t L = 0, pre = 0;
-#pragma unroll
-    for (int w = 0; w < 8; ++w) { L += s_red[0][w]; pre += s_red[1][w]; }
 
-    // the decision (identical in every CTA of the unit)
-    bool ok;
-    int64_t base = 0, head = head0, oldest = oldest0, nf = nf0;
-    if (is_cond) {
-        ok = ncond0 < bk.n_cond && cond_len0 + L <= bk.pinned_cap;
-        base = cond_len0;
-    } else {
-        const bool sane = head0 >= 0 && tail0 >= head0 && nf0 >= 0 && nf0 <= bk.max_frames &&
-                          oldest0 >= 0 && oldest0 < bk.max_frames;
-        if (!sane) {
-            if (threadIdx.x == 0 && ch == 0) latch_status(status, RS3_EINTERNAL);
-            ok = false;
+    // ranks of the chunk's kept cells, in cell order
+    const uint32_t bal = __ballot_sync(0xffffffffu, keep);
+    if (lane == 0) s_wc[warp] = __popc(bal);
+    __syncthreads();
+    int off = 0, nk = 0;
+#pragma unroll
+    for (int w = 0; w < NW; ++w) {
+        off += w < warp ? s_wc[w] : 0;
+        nk += s_wc[w];
+    }
+    if (keep) {
+        uint32_t lm;
+        asm("mov.u32 %0, %%lanemask_lt;" : "=r"(lm));
+        s_list[off + __popc(bal & lm)] = cell;
+    }
+    __syncthreads();
+
+    // round trip 2: the first batch of the chunk's rows in flight ...
+    const int nvec = (int)(row_bytes / 16);
+    const uint8_t *ksrc = k_new + (size_t)u * mn * row_bytes;
+    const uint8_t *vsrc = v_new + (size_t)u * mn * row_bytes;
+    uint4 kk[COMMIT_PF], vv[COMMIT_PF];
+    commit_load<NW>(kk, vv, s_list, nk, warp, lane, nvec, ksrc, vsrc, row_bytes);
+
+    // ... while the unit's counts are summed and thread 0 decides
+    if (Mu) {
+        total = warp_sum(total);
+        before = warp_sum(before);
+        if (lane == 0) { s_red[0][warp] = total; s_red[1][warp] = before; }
+    }
+    __syncthreads();
+    bool ok = false;
+    int64_t L = 0, head = head0, oldest = oldest0, nf = nf0;
+    if (threadIdx.x == 0) {
+        int64_t pre = 0;
+        if (Mu) {
+#pragma unroll
+            for (int w = 0; w < NW; ++w) { L += s_red[0][w]; pre += s_red[1][w]; }
         } else {
-            if (bk.window > 0 && nf == bk.window) {      // evict the oldest ring frame
-                head += flen[oldest];
-                oldest = (oldest + 1) % bk.max_frames;
-                nf -= 1;
-            }
-            ok = nf < bk.max_frames && (tail0 - head) + L <= bk.ring_cap;
-            base = tail0;
+            L = mn;
+            pre = c0;
         }
-    }
-
-    if (ok) {
-        // ranks of the kept cells of this chunk (ballot / popc), then copies
-        const int cell = ch * COMMIT_CHUNK + threadIdx.x;
-        const bool keep = threadIdx.x < COMMIT_CHUNK && cell < mn && (Mu ? Mu[cell] != 0 : true);
-        const uint32_t bal = __ballot_sync(0xffffffffu, keep);
-        __syncthreads();
-        if (lane == 0) s_red[0][warp] = __popc(bal);
-        __syncthreads();
-        int off = 0, nk = 0;
-#pragma unroll
-        for (int w = 0; w < 8; ++w) {
-            off += (w < warp) ? s_red[0][w] : 0;
-            nk += s_red[0][w];
-        }
-        if (keep) {
-            uint32_t lm;
-            asm("mov.u32 %0, %%lanemask_lt;" : "=r"(lm));
-            const int j = off + __popc(bal & lm);
-            const int64_t rank = pre + j;
-            s_list[j] = cell;
-            s_row[j] = is_cond ? base + rank : bk.pinned_cap + (base + rank) % bk.ring_cap;
-        }
-        __syncthreads();
-        // the chunk's rows as 16-byte pieces over all threads, four pieces'
-        // K and V loads in flight before their stores
-        const int nvec = (int)(row_bytes / 16);
-        const int npiece = nk * nvec;
-        const uint8_t *ksrc = k_new + (size_t)u * mn * row_bytes;
-        const uint8_t *vsrc = v_new + (size_t)u * mn * row_bytes;
-        uint8_t *kdst = k_store + (size_t)u * bk.rows_per_unit * row_bytes;
-        uint8_t *vdst = v_store + (size_t)u * bk.rows_per_unit * row_bytes;
-        for (int i0 = threadIdx.x; i0 < npiece; i0 += 4 * blockDim.x) {
-            uint4 kk[4], vv[4];
-            int64_t dst[4];
-            int cellq[4], eq[4];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int i = i0 + q * blockDim.x;
-                if (i < npiece) {
-                    const int j = i / nvec, v = i - j * nvec;
-                    const int64_t so = (int64_t)s_list[j] * row_bytes + 16 * v;
-                    dst[q] = s_row[j] * row_bytes + 16 * v;
-                    cellq[q] = s_list[j];
-                    eq[q] = (16 * v) / esz;                  // first element of the piece
-                    kk[q] = __ldcs(reinterpret_cast<const uint4 *>(ksrc + so));
-                    vv[q] = __ldcs(reinterpret_cast<const uint4 *>(vsrc + so));
+        int64_t row0 = 0;
+        if (is_cond) {
+            ok = ncond0 < bk.n_cond && cond_len0 + L <= bk.pinned_cap;
+            row0 = cond_len0 + pre;
+        } else {
+            const bool sane = head0 >= 0 && tail0 >= head0 && nf0 >= 0 && nf0 <= bk.max_frames &&
+                              oldest0 >= 0 && oldest0 < bk.max_frames;
+            if (!sane) {
+                if (ch == 0) latch_status(status, RS3_EINTERNAL);
+            } else {
+                if (bk.window > 0 && nf == bk.window) {      // evict the oldest ring frame
+                    head += mu[BM_HEADER_WORDS + bk.max_frames + oldest];
+                    oldest = oldest + 1 == bk.max_frames ? 0 : oldest + 1;
+                    nf -= 1;
                 }
-            }
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                if (i0 + q * (int)blockDim.x < npiece) {
-                    if (rope)                              // keys stored rotated by their own cell
-                        kk[q] = rotate_piece(kk[q], rope + ((int64_t)cellq[q] * (d / 2) + (eq[q] % d) / 2) * 2,
-                                             esz);
-                    *reinterpret_cast<uint4 *>(kdst + dst[q]) = kk[q];
-                    *reinterpret_cast<uint4 *>(vdst + dst[q]) = vv[q];
-                }
+                ok = nf < bk.max_frames && (tail0 - head) + L <= bk.ring_cap;
+                if (ok && L > 0) row0 = (tail0 + pre) % bk.ring_cap;   // it fits: rows wrap at most once
             }
         }
+        s_ok = ok;
+        s_row0 = row0;
     }
-
-    // arrival; the last CTA of the unit publishes the new counters
     __syncthreads();
+
+    // every read of the old counters by this CTA is done: arrive
+    unsigned long long arrived = 0;
     if (threadIdx.x == 0) {
         __threadfence();
-        unsigned long long *arrive = reinterpret_cast<unsigned long long *>(mu + BM_ARRIVE);
-        s_last = atomicAdd(arrive, 1ull) == (unsigned long long)(gridDim.x - 1);
+        arrived = atomicAdd(reinterpret_cast<unsigned long long *>(mu + BM_ARRIVE), 1ull);
     }
-    __syncthreads();
-    if (!s_last || threadIdx.x != 0) return;
+
+    if (s_ok) {
+        const int64_t row0 = s_row0;
+        uint8_t *kdst = k_store + (size_t)u * bk.rows_per_unit * row_bytes;
+        uint8_t *vdst = v_store + (size_t)u * bk.rows_per_unit * row_bytes;
+        commit_store<NW, ROPE>(kk, vv, s_list, nk, warp, lane, nvec, row0, is_cond, bk, kdst, vdst,
+                               row_bytes, rope, d, esz);
+        // the rest of the chunk (rows past the first batch, pieces past 32 per row)
+        for (int vb = 0; vb < nvec; vb += 32) {
+            for (int jb = vb == 0 ? NW * COMMIT_PF : 0; jb < nk; jb += NW * COMMIT_PF) {
+                commit_load<NW>(kk, vv, s_list, nk, jb + warp, vb + lane, nvec, ksrc, vsrc, row_bytes);
+                commit_store<NW, ROPE>(kk, vv, s_list, nk, jb + warp, vb + lane, nvec, row0, is_cond, bk, kdst,
+                                       vdst, row_bytes, rope, d, esz);
+            }
+        }
+    }
+
+    // the last CTA of the unit to arrive publishes the new counters
+    if (threadIdx.x != 0 || arrived != (unsigned long long)(gridDim.x - 1)) return;
     __threadfence();
     mu[BM_ARRIVE] = 0;
     if (!ok) {
@@ -356,9 +408,16 @@ rs3_status commit_launch(const rs3_bank *bank, const void *k_new, const void *v_
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const BankDev bk = bank_dev(bank);
     const int mn = bank->mn;
-    const int nchunks = (mn + COMMIT_CHUNK - 1) / COMMIT_CHUNK;
     const int64_t row_bytes = (int64_t)bank->D * (int64_t)elem_bytes(bank->dtype);
-    launch_pdl(k_commit, dim3(nchunks, bank->U), dim3(256), 0, st,
+    // 128-cell chunks, or 64-cell ones where those would give under two CTAs per SM
+    const bool small = (int64_t)((mn + 127) / 128) * bank->U < 2ll * rs3_sm_count();
+    const int chunk = small ? 64 : 128;
+    const dim3 grid((unsigned)((mn + chunk - 1) / chunk), (unsigned)bank->U);
+    void (*kern)(const uint8_t *, const uint8_t *, const uint8_t *, int, int, int64_t, BankDev, uint8_t *,
+                 uint8_t *, int32_t *, const float *, int, int) =
+        small ? (rope ? k_commit<64, true> : k_commit<64, false>)
+              : (rope ? k_commit<128, true> : k_commit<128, false>);
+    launch_pdl(kern, grid, dim3(chunk), 0, st,
         static_cast<const uint8_t *>(k_new), static_cast<const uint8_t *>(v_new), keep_mask, mn, is_cond,
         row_bytes, bk, static_cast<uint8_t *>(bank->k_store), static_cast<uint8_t *>(bank->v_store), status,
         rope, bank->d, elem_bytes(bank->dtype));

@@ -24,7 +24,7 @@ enum {
     BM_OLDEST = 4,      // frame-table slot of the oldest ring frame
     BM_NCOND = 5,       // pinned frames held
     BM_PTRLEN = 6,      // pointer rows held
-    BM_ARRIVE = 8,      // CTAs of the running commit that have finished
+    BM_ARRIVE = 8,      // CTAs of the running commit that have read the old counters
     BM_HEADER_WORDS = 16
 };
 // after the header: int64 foff[max_frames], int64 flen[max_frames]
@@ -33,8 +33,6 @@ __host__ __device__ inline int64_t bank_meta_words(int max_frames)
 {
     return (int64_t)BM_HEADER_WORDS + 2 * (int64_t)max_frames;
 }
-
-#define COMMIT_CHUNK 128
 
 // ---------------------------------------------------------------------------
 // Readout work list (in the caller's workspace)

@@ -19,11 +19,14 @@ def test_frame_work_closed_form():
     counts = [1228, 600, 0, 5, 1228, 1000, 1, 300]
     banks = [5000, 4000, 7000, 0, 100, 6000, 28672, 16]
     kw = [800, 0, 1600, 4096, 10, 20, 30, 40]
-    flops, cbytes = bench.frame_work(w, counts, banks, kw)
+    flops, cbytes, sbytes = bench.frame_work(w, counts, banks, kw)
     # Eq. 6 per unit: q~ K^T and P V, each 2 |K_r| N d flops per head
     assert flops == sum(4.0 * c * n * w.H * w.d for c, n in zip(counts, banks))
     # commit: every unit's mask, K and V rows read and written (bf16)
     assert cbytes == w.U * w.mn + sum(4 * L * w.D * 2 for L in kw)
+    # selection: the group's grid z, each unit's previous mask, the keep-set
+    # indices and counts written, the tracker state (6 int32) read and written
+    assert sbytes == w.G * w.mn * w.D * 2 + w.U * w.mn + 4 * sum(counts) + 4 * w.U + 2 * 6 * 4 * w.U
 
 
 def test_traffic_key_ignores_comments_not_code(tmp_path, monkeypatch):
