@@ -106,8 +106,17 @@ k_prior(const uint8_t *__restrict__ masks, int m, int n, const int32_t *__restri
     uint8_t *sT = smem + ((mn + 15) & ~15);
     __shared__ int s_mode, s_r, s_g, s_box[4];
 
+    // the unit's group and tracker state load beside the mask (thread 0
+    // decides the prior's mode once the mask's box is known)
+    int g0 = 0;
+    rs3_track t0 = {};
+    if (threadIdx.x == 0) {
+        g0 = unit_group[u];
+        t0 = track[u];
+    }
     const uint8_t *Mu = masks + (size_t)u * mn;
     int y0 = INT_MAX, x0 = INT_MAX, y1 = -1, x1 = -1;
+#pragma unroll 4
     for (int i = threadIdx.x; i < mn; i += blockDim.x) {
         const uint8_t v = Mu[i] != 0;
         sM[i] = v;
@@ -120,8 +129,8 @@ k_prior(const uint8_t *__restrict__ masks, int m, int n, const int32_t *__restri
     block_bbox(y0, x0, y1, x1);   // contains __syncthreads
 
     if (threadIdx.x == 0) {
-        const int g = unit_group[u];
-        rs3_track t = track[u];
+        const int g = g0;
+        rs3_track t = t0;
         int mode, r = 0;
         if (g < 0 || g >= G) {
             latch_status(status, RS3_EINVAL);
@@ -293,10 +302,15 @@ k_select(const uint8_t *__restrict__ prior, const uint32_t *__restrict__ need,
     const uint8_t *Pu = prior + (size_t)u * mn;
     const uint32_t *Ng = need + (size_t)g * nwords;
     const float *eg = e + (size_t)g * mn;
+    // every load of the loop is independent (the energy is read whether or
+    // not the cell is in the prior: the buffer holds mn values per group), so
+    // the unrolled iterations share one round trip
     uint32_t np_local = 0;
+#pragma unroll 4
     for (int i = threadIdx.x; i < mn; i += blockDim.x) {
+        const uint32_t ebits = __float_as_uint(eg[i]);
         const bool inP = union_mode ? ((Ng[i >> 5] >> (i & 31)) & 1u) : (Pu[i] != 0);
-        skey[i] = inP ? __float_as_uint(eg[i]) : KEY_NONE;
+        skey[i] = inP ? ebits : KEY_NONE;
         np_local += inP ? 1u : 0u;
     }
     uint32_t nP;
