@@ -81,3 +81,63 @@ def test_close_argmax_work_closed_form():
     assert bench.close_argmax_work(w) == 8 * 256 * 256 * 4 + 256 * 256 + 8 * 64 * 64
     w = synth.WORKLOADS["multistream"]
     assert bench.close_argmax_work(w) == 48 * 384 * 384 * 4 + 16 * 384 * 384 + 48 * 96 * 96
+
+
+class _Rec:
+    """Stands in for the pipeline and the device inputs: records the calls."""
+
+    def __init__(self, w):
+        self.w = w
+        self.calls = []
+        self.track = self
+        self.bank = None
+
+    def zero_(self):
+        self.calls.append(("track_zero",))
+
+    def use_buffer(self, i):
+        self.calls.append(("buffer", i))
+
+    def select(self, z, prev, stream=None):
+        self.calls.append(("select", z[1], prev[1]))
+
+    def commit(self, k, v, mask, is_cond, rope=None):
+        self.calls.append(("commit", k[1], None if mask is None else mask[1], is_cond))
+
+
+class _Data:
+    def __init__(self, w):
+        self.T = w.frames + w.prefill_frames
+        self.P = w.prefill_frames
+        self.rope = None
+
+    @staticmethod
+    def frame(key, t):
+        return (key, t)
+
+
+@pytest.mark.parametrize("name", sorted(synth.WORKLOADS))
+def test_per_call_graphs_issue_the_pass_calls(name, monkeypatch):
+    """The per-call times divide graphs of one kind of call by the readout
+    frames: "select" holds one selection per readout frame (on its keep-set
+    buffer), "commit" every commit of the pass in order, "setup" the commits
+    before the first readout frame, so commit minus setup is one commit per
+    readout frame."""
+    from paper_2608_22526_gb300 import rs3
+    monkeypatch.setattr(rs3, "rs3_bank_reset", lambda *a, **k: None)
+    w = synth.WORKLOADS[name]
+    data = _Data(w)
+    first = data.P + (1 if w.n_cond > 0 else 0)
+    readout = list(range(first, data.T))
+    out = {}
+    for what in ("select", "commit", "setup"):
+        pipe = _Rec(w)
+        bench.calls_only(pipe, data, what)
+        out[what] = [c for c in pipe.calls if c[0] != "track_zero"]
+    sel = out["select"]
+    assert sel == [c for t in readout for c in (("buffer", t % 2), ("select", t, t))]
+    setup = [("commit", t, None, 0) for t in range(data.P)]
+    if w.n_cond > 0:
+        setup.append(("commit", data.P, data.P, 1))
+    assert out["setup"] == setup
+    assert out["commit"] == setup + [("commit", t, t, 0) for t in readout]
