@@ -113,9 +113,6 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // another stream could use.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-// Lets the next kernel of the stream launch now (its pdl_wait() still waits
-// for this kernel to finish and its writes to be visible).
-__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 template <typename... KArgs, typename... Args>
 inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
