@@ -218,7 +218,8 @@ typedef struct {
 /* Sizes for a bank: rows per unit of each store and bytes of meta.
  * window > 0 requires ring_cap_rows >= window * mn (the ring then always holds
  * the window); window == -1 (unbounded) needs ring_cap_rows >= 0 and
- * max_frames >= 1.  Returns RS3_EINVAL on an inconsistent layout. */
+ * max_frames >= 1.  Returns RS3_EINVAL on an inconsistent layout and
+ * RS3_EUNSUPPORTED for mn > 16384 or U > 65535. */
 rs3_status rs3_bank_layout(int U, int H, int d, rs3_dtype dtype, int mn, int n_cond, int window,
                            int64_t ring_cap_rows, int max_frames, int n_ptr,
                            int64_t *rows_per_unit, size_t *meta_bytes);

@@ -351,6 +351,7 @@ extern "C" rs3_status rs3_bank_layout(int U, int H, int d, rs3_dtype dtype, int 
         return RS3_EINVAL;
     if (dtype != RS3_F32 && dtype != RS3_BF16) return RS3_EINVAL;
     if (mn > RS3_MAX_MN) return RS3_EUNSUPPORTED;
+    if (U > 65535) return RS3_EUNSUPPORTED;          // a commit's grid holds a row of CTAs per unit
     if (((int64_t)H * d * (int64_t)elem_bytes(dtype)) % 16 != 0) return RS3_EINVAL;
     if (window == 0 || window < -1) return RS3_EINVAL;
     if (window > 0) {

@@ -73,9 +73,12 @@ def test_bank_layout_rules(binding):
         with pytest.raises(binding.RS3Error) as e:
             binding.rs3_bank_layout(*args)
         assert e.value.code == binding.RS3_EINVAL
-    with pytest.raises(binding.RS3Error) as e:
-        binding.rs3_bank_layout(1, 1, 64, "bf16", 20000, 0, -1, 10, 4, 0)
-    assert e.value.code == binding.RS3_EUNSUPPORTED
+    for args in [(1, 1, 64, "bf16", 20000, 0, -1, 10, 4, 0),     # mn above 16384
+                 (65536, 1, 64, "bf16", 16, 0, -1, 16, 1, 0)]:    # more units than a grid column
+        with pytest.raises(binding.RS3Error) as e:
+            binding.rs3_bank_layout(*args)
+        assert e.value.code == binding.RS3_EUNSUPPORTED
+    assert binding.rs3_bank_layout(65535, 1, 64, "bf16", 16, 0, -1, 16, 1, 0)[0] == 16
 
 
 def test_workspace_sizes(binding):
